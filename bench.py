@@ -1,0 +1,385 @@
+"""Benchmark of the budget-routed decode step (one JSON line on stdout).
+
+python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                [--workload NAME] [--no-graph]
+
+Default workload: Llama-3-8B shape, bf16, batch 1, context 2048, budget k = 15
+of 30 middle layers (the configuration the headline metric is quoted on).
+A step = one budget-routed decode step of the whole batch (layer 0, router,
+compaction, the selected middle layers on their sub-batches, last layer).
+Inputs (weights 14 GB, KV cache) are resident in HBM and larger than L2.
+
+For N > 1 (torchrun) every rank runs an independent replica of the workload on
+its own GPU (weak scaling); the only cross-rank traffic is a barrier and the
+max-over-ranks of the timed region.  `--impl reference` times the CPU oracle
+on the host cores instead (rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "budget-routed decode tokens/s at 1 GB300 per budget; % of HBM/tensor roofline"
+# ncu dram bytes per launch of the dominant kernel, from the committed profile
+# summary of the current kernel (None until captured for this kernel version)
+NCU_TRAFFIC_PER_LAUNCH = {}
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return 6800.0, 1700.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "20"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.out = ""
+        if self.proc is not None:
+            time.sleep(0.1)
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        for line in (self.out or "").strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                rows.append((float(f[1]), float(f[2]), f[5:9]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        mx = max(r[1] for r in rows)
+        load = [r for r in rows if r[0] > 0.5 * mx] or rows
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[j] for r in rows for j in range(4) if r[2][j].lower() == "active"})
+        return {"sm_mhz": float(np.median([r[0] for r in load])), "sm_max_mhz": mx,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def _max_over_ranks(x: float, ws: int, device) -> float:
+    if ws == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def _barrier(ws: int):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle sample (cpu_baseline and the reference arm)
+# ---------------------------------------------------------------------------
+def oracle_sample(w, n_layers_sample=None, steps=1, device="cuda"):
+    """Times the oracle on one sequence of the workload for `steps` decode
+    steps.  Weights/KV come from the shared generator (generated on `device`
+    and copied to host; that preparation is excluded).  If n_layers_sample is
+    given, each step runs layer 0, the router, the first n_layers_sample
+    selected middle layers and the last layer, and the time is scaled to the
+    full routed depth."""
+    import torch
+
+    from oracle import adapter as A
+    from oracle import buddy_oracle as O
+    from workloads import synth
+
+    s = w.shape
+    seq = 0
+    prep = {"t": 0.0}
+
+    def src(l):
+        t0 = time.perf_counter()
+        out = {k: v.cpu() for k, v in synth.layer_weights(s, w.seed, l, device).items()}
+        prep["t"] += time.perf_counter() - t0
+        return out
+
+    model = A.build_model(s, w.seed, layer_source=src,
+                          dm_source=lambda: {k: v.cpu() for k, v in synth.dm_weights(s, w.seed, device).items()},
+                          cache_layers=2)
+    t0 = time.perf_counter()
+    st = A.build_state(s, w.seed, [int(w.contexts()[seq])], seqs=[0], gen_device=device)
+    prep["t"] += time.perf_counter() - t0
+    k = [int(w.budgets()[seq])]
+    total = 0.0
+    scaled_total = 0.0
+    for t in range(steps):
+        h = A.to_f64(synth.h_in(s, w.seed, t, [seq], device))
+        prep0 = prep["t"]
+        t0 = time.perf_counter()
+        route = O.first_layer_and_route(model, st, h, k)
+        if n_layers_sample is not None:
+            keep = route.sel[0][:n_layers_sample]
+            full = len(route.sel[0])
+            route.sel = [keep]
+        res = O.routed_layers(model, st, route)
+        O.advance(st, res)
+        dt = time.perf_counter() - t0 - (prep["t"] - prep0)
+        total += dt
+        if n_layers_sample is not None:
+            scaled_total += dt * (full + 2) / (len(keep) + 2)
+        else:
+            scaled_total += dt
+    return {"seconds": total, "scaled_seconds": scaled_total, "tokens": steps,
+            "cores": os.cpu_count()}
+
+
+# ---------------------------------------------------------------------------
+# Our arm
+# ---------------------------------------------------------------------------
+def run_ours(args, ws, rank, local):
+    import torch
+
+    from workloads import configs as C
+    from workloads import cost
+    from workloads import device as D
+    from workloads import synth
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    w = C.BY_NAME[args.workload]
+    s = w.shape
+    B = w.batch
+    K, W = args.steps, args.warmup
+    prof_steps = min(K, 8)
+    e2e_steps = K
+    extra = W + K + prof_steps + e2e_steps + 2
+    dw = D.build(w, device=dev, extra_steps=extra, use_graph=not args.no_graph)
+    ctx, kv = dw.ctx, dw.kv
+    n_steps_total = W + K + prof_steps + e2e_steps
+    h_all = [synth.h_in(s, w.seed, t, range(B), dev) for t in range(n_steps_total)]
+    h_out = torch.empty(B, s.d_model, device=dev)
+    count = torch.empty(s.n_layers, dtype=torch.int32, device=dev)
+    mask = torch.empty(B, s.n_layers, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    # warm-up (also captures the graph)
+    step = 0
+    for _ in range(W):
+        ctx.buddy_decode_step(kv, h_all[step], dw.k, h_out, mask, None, count)
+        step += 1
+    torch.cuda.synchronize(dev)
+    if ctx.buddy_device_status() != 0:
+        raise RuntimeError("device error flag during warm-up")
+
+    # timed region: K steps, positions advancing
+    n_ctx_timed = []
+    masks = []
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        _barrier(ws)
+        torch.cuda.synchronize(dev)
+        lens0 = kv.len.cpu().numpy().copy()
+        start.record(stream)
+        for t in range(K):
+            ctx.buddy_decode_step(kv, h_all[step], dw.k, h_out, mask, None, count)
+            step += 1
+        end.record(stream)
+        torch.cuda.synchronize(dev)
+        _barrier(ws)
+    ms = start.elapsed_time(end)
+    ms_max = _max_over_ranks(ms, ws, dev)
+    if ctx.buddy_device_status() != 0:
+        raise RuntimeError("device error flag in timed region")
+
+    # instrumented pass: per-kernel-class CUDA events (direct launches)
+    ctx.buddy_set_options(False)
+    ctx.buddy_set_profiling(True)
+    ctx.buddy_profile_read()
+    prof_masks, prof_ctx = [], []
+    for t in range(prof_steps):
+        prof_ctx.append(kv.len.cpu().numpy().copy())
+        ctx.buddy_decode_step(kv, h_all[step], dw.k, h_out, mask, None, count)
+        torch.cuda.synchronize(dev)
+        prof_masks.append(mask.cpu().numpy().copy())
+        step += 1
+    prof = ctx.buddy_profile_read()
+    ctx.buddy_set_profiling(False)
+    ctx.buddy_set_options(not args.no_graph)
+
+    # end to end through the host-buffer entry point (pinned buffers)
+    h_host = [h.cpu().pin_memory() for h in h_all[step:step + e2e_steps]]
+    k_host = dw.k.cpu().pin_memory()
+    o_host = torch.empty(B, s.d_model).pin_memory()
+    m_host = torch.empty(B, s.n_layers, dtype=torch.uint8).pin_memory()
+    ctx.buddy_decode_step_host(kv, h_host[0], k_host, o_host, m_host)   # graph for the staging buffers
+    step += 1
+    _barrier(ws)
+    t0 = time.perf_counter()
+    for t in range(1, e2e_steps):
+        ctx.buddy_decode_step_host(kv, h_host[t], k_host, o_host, m_host)
+    e2e_s = time.perf_counter() - t0
+    e2e_s = _max_over_ranks(e2e_s, ws, dev)
+    e2e_n = e2e_steps - 1
+
+    # algorithmic cost of the profiled steps (realised masks and lengths)
+    hbm, tflops, peak_src = _peaks()
+    c_sum = {"bytes": 0, "flops": 0, "weight_bytes": 0, "kv_read_bytes": 0}
+    for m_, n_ in zip(prof_masks, prof_ctx):
+        c = cost.step_cost(s, m_, n_[:B])
+        for key in c_sum:
+            c_sum[key] += c[key]
+    prof_ms_total = sum(v[0] for v in prof.values())
+    # dominant kernel class and its algorithmic bytes per launch
+    dom = max(prof, key=lambda k: prof[k][0])
+    esz = s.elem_bytes
+    rows_per_layer = [m_.sum(axis=0) for m_ in prof_masks]
+    exec_layers = [(r > 0) for r in rows_per_layer]
+    n_launch_layers = int(sum(e.sum() for e in exec_layers))
+    m_sum = int(sum(r.sum() for r in rows_per_layer))
+    per_class_bytes = {
+        "gemm_gate_up": 2 * s.ffn_dim * s.d_model * esz * n_launch_layers + m_sum * (s.d_model + s.ffn_dim) * esz,
+        "gemm_down": s.ffn_dim * s.d_model * esz * n_launch_layers + m_sum * (s.ffn_dim * esz + 8 * s.d_model),
+        "gemm_qkv": s.qkv_dim * s.d_model * esz * n_launch_layers + m_sum * (s.d_model * esz + 4 * s.qkv_dim),
+        "gemm_o": s.q_dim * s.d_model * esz * n_launch_layers + m_sum * (s.q_dim * esz + 8 * s.d_model),
+    }
+    roof = None
+    if dom in per_class_bytes and prof[dom][1] > 0:
+        launches = prof[dom][1]
+        bytes_per_launch = per_class_bytes[dom] / launches
+        avg_s = prof[dom][0] / 1e3 / launches
+        ach = bytes_per_launch / avg_s / 1e9
+        roof = {"bound": "hbm", "kernel": dom, "achieved": round(ach, 1), "peak": hbm, "unit": "GB/s",
+                "frac": round(ach / hbm, 4), "traffic": NCU_TRAFFIC_PER_LAUNCH.get(dom),
+                "bytes_per_launch": int(bytes_per_launch), "avg_launch_us": round(avg_s * 1e6, 2),
+                "launches": launches, "peak_source": f"{peak_src} hbm_gbs"}
+    t_roof = max(c_sum["bytes"] / (hbm * 1e9), c_sum["flops"] / (tflops * 1e12)) / prof_steps
+    step_s = ms_max / 1e3 / K
+    route_frac = (prof["route"][0] + prof["compact"][0]) / max(prof_ms_total, 1e-9)
+    launches_per_step = sum(v[1] for v in prof.values()) / prof_steps
+    graph_extra = (s.n_layers - 2) if not args.no_graph else 0   # conditional-setting kernels
+    value = ws * B * K / (ms_max / 1e3)
+    out = {
+        "metric": METRIC, "value": round(value, 2), "unit": "tokens/s", "n_gpus": ws, "steps": K,
+        "warmup": W, "ms_per_step": round(ms_max / K, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": s.dtype, "data": "synthetic (seeded counter-based generator)",
+        "config": {"workload": w.name, "model": s.name, "batch": B, "ctx": w.ctx_args,
+                   "k": w.k_args, "layers": s.n_layers, "parallelism": f"replicas x{ws}",
+                   "graph": not args.no_graph,
+                   "l2": "inputs larger than L2 (per-step weight stream %.1f GB)" % (c_sum["weight_bytes"] / prof_steps / 1e9)},
+        "roofline": roof,
+        "step_roofline": {"t_roof_ms": round(t_roof * 1e3, 4), "frac": round(t_roof / step_s, 4),
+                          "bytes_per_step": int(c_sum["bytes"] / prof_steps),
+                          "flops_per_step": int(c_sum["flops"] / prof_steps), "peak_gbs": hbm,
+                          "peak_source": peak_src},
+        "route_compact_frac": round(route_frac, 4),
+        "kernel_ms_per_step": {k: round(v[0] / prof_steps, 4) for k, v in prof.items()},
+        "e2e": {"value": round(ws * B * e2e_n / e2e_s, 2), "unit": "tokens/s",
+                "h2d_bytes_per_step": B * s.d_model * 4 + B * 4,
+                "d2h_bytes_per_step": B * s.d_model * 4 + B * s.n_layers},
+        "gpu_launches": int(round((launches_per_step + graph_extra) * K)),
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and not args.no_cpu:
+        o = oracle_sample(w, n_layers_sample=None, steps=1, device=dev)
+        out["cpu_baseline"] = {"value": round(o["tokens"] / o["scaled_seconds"], 5), "unit": "tokens/s",
+                               "cores": o["cores"], "kind": "oracle",
+                               "sample": f"1 decode step of sequence 0 of {w.name} (numpy float64; "
+                                         f"weight generation and host copy excluded)"}
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    ctx.close()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def run_reference(args, ws, rank, local):
+    if rank != 0:
+        return
+    import torch
+    from workloads import configs as C
+    w = C.BY_NAME[args.workload]
+    dev = torch.device("cuda", local) if torch.cuda.is_available() else "cpu"
+    # bounded per-step sample: layer 0, router, 1 selected middle layer, last layer,
+    # time scaled to the full routed depth
+    o = oracle_sample(w, n_layers_sample=1, steps=args.warmup + args.steps, device=dev)
+    per_tok = o["scaled_seconds"] / o["tokens"]
+    value = 1.0 / per_tok
+    out = {"metric": METRIC, "value": round(value, 5), "unit": "tokens/s", "n_gpus": 1, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": round(per_tok * 1e3, 2), "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "impl": "reference",
+           "config": {"workload": w.name, "model": w.shape.name, "batch": w.batch},
+           "cpu_baseline": {"value": round(value, 5), "unit": "tokens/s", "cores": o["cores"], "kind": "oracle",
+                            "sample": "per step: sequence 0 through layer 0, router, the first selected "
+                                      "middle layer and the last layer; time scaled by routed depth"},
+           "e2e": {"value": round(value, 5), "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=64)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama3-8b-b1")
+    ap.add_argument("--no-graph", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline oracle sample")
+    args = ap.parse_args()
+    ws, rank, local = _dist()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args, ws, rank, local)
+    else:
+        run_ours(args, ws, rank, local)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,227 @@
+/*
+ * libbuddy — budget-routed batched decode (BUDDY, arXiv 2606.09514) on one
+ * NVIDIA GB300 (sm_103a).
+ *
+ * One decode step, for every sequence i of a batch:
+ *   1. runs the first decoder block (always executed, Sec. 4.2.1);
+ *   2. pools the first layer's value cache, including the newest token, and
+ *      concatenates the newest token's hidden state (KV-aware planner, Sec. 4.3);
+ *   3. scores the L-2 middle blocks with the Decision Module, a
+ *      Linear-SiLU-Linear MLP (App. C.1), fused with an optional prior
+ *      s' = s + omega * p~ (Eq. 2);
+ *   4. executes the k_i highest-scoring middle blocks (Eq. 2, ties to the lower
+ *      layer index), each block on the sub-batch of sequences that selected it
+ *      (grouping by mask, App. C.1), skipped blocks being the identity (Eq. 1)
+ *      and storing zero K/V at the new position (Sec. 6);
+ *   5. runs the last block (always executed) and advances every sequence's
+ *      position by one (KV cache update, Eq. 9).
+ *
+ * Conventions for every entry point:
+ *   - Pointers marked "device" are device pointers owned by the caller; the
+ *     library never frees them.  Weight pointers are retained (not copied) by
+ *     buddy_set_weights and must stay valid while the context is used.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *     Calls are asynchronous on that stream unless stated otherwise.
+ *   - Return value: BUDDY_OK or a BUDDY_ERR_* code.  On a host-detected error
+ *     nothing is launched and nothing is written.  Conditions that only the
+ *     device can see (a budget or position stored in device memory out of
+ *     range) make every kernel of that call return without writing; the flag
+ *     is reported by buddy_device_status().
+ *   - The library allocates device memory only in buddy_create (scratch sized
+ *     by max_batch and max_pos) and in buddy_set_weights (tensor descriptors).
+ */
+#ifndef BUDDY_H_
+#define BUDDY_H_
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define BUDDY_API __attribute__((visibility("default")))
+#else
+#define BUDDY_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+  BUDDY_OK = 0,
+  BUDDY_ERR_ARG = 1,      /* null pointer, bad size, unsupported shape */
+  BUDDY_ERR_RANGE = 2,    /* value outside its documented range (host-visible) */
+  BUDDY_ERR_CUDA = 3,     /* a CUDA runtime call failed */
+  BUDDY_ERR_DEVICE = 4,   /* a kernel raised the device error flag */
+  BUDDY_ERR_STATE = 5     /* call order: e.g. weights not set */
+};
+
+enum { BUDDY_DTYPE_F32 = 0, BUDDY_DTYPE_BF16 = 1 };
+
+/* Bits of the device error flag (buddy_device_status). */
+enum {
+  BUDDY_DEV_BAD_BUDGET = 1,    /* k_i outside [1, L-2] */
+  BUDDY_DEV_BAD_POSITION = 2,  /* len_i + new positions > cap_i or > max_pos */
+  BUDDY_DEV_BAD_SEQ = 4,       /* a sequence id outside [0, batch) */
+  BUDDY_DEV_TIMEOUT = 8        /* a bounded wait inside a kernel ran out */
+};
+
+typedef struct buddy_ctx buddy_ctx;
+
+/* Model shape.  The decoder block is Llama-style (App. "Background"):
+ * RMSNorm, Q/K/V projections (optional bias, Qwen2.5), rotate-half RoPE,
+ * grouped-query attention, output projection, RMSNorm, SwiGLU MLP d->F->d.
+ * Requirements: n_layers >= 3; head_dim 64 or 128; n_q_heads a multiple of
+ * n_kv_heads (group of at most 8); d_model == n_q_heads * head_dim; ffn_dim a
+ * multiple of 8; dm_hidden >= 1; 1 <= max_batch <= 1024; max_pos >= 1. */
+typedef struct {
+  int32_t n_layers;     /* L */
+  int32_t d_model;      /* d */
+  int32_t n_q_heads;
+  int32_t n_kv_heads;
+  int32_t head_dim;
+  int32_t ffn_dim;      /* F */
+  int32_t dm_hidden;    /* r: Decision Module hidden width */
+  int32_t dtype;        /* BUDDY_DTYPE_F32 or BUDDY_DTYPE_BF16: weights, KV cache, GEMM inputs */
+  int32_t max_batch;    /* largest B of any call */
+  int32_t max_pos;      /* every position p written or read satisfies p < max_pos */
+  int32_t qkv_bias;     /* 1: Q/K/V projections carry a bias */
+  float rms_eps;
+  float rope_theta;
+} buddy_config;
+
+/* One decoder layer; matrices row-major in nn.Linear layout [out, in],
+ * element type = config dtype; gains and biases fp32. */
+typedef struct {
+  const float* attn_norm;   /* device [d] */
+  const void* w_qkv;        /* device [(n_q + 2 n_kv) * hd, d]: Q rows, then K rows, then V rows */
+  const float* b_qkv;       /* device [(n_q + 2 n_kv) * hd], or NULL when qkv_bias == 0 */
+  const void* w_o;          /* device [d, n_q * hd] */
+  const float* ffn_norm;    /* device [d] */
+  const void* w_gate_up;    /* device [2F, d]: rows [0, F) gate, rows [F, 2F) up */
+  const void* w_down;       /* device [d, F] */
+} buddy_layer_weights;
+
+/* Decision Module (App. C.1): s' = W2 SiLU(W1 x + b1) + b2 + omega * prior,
+ * x = [pool expanded to d ; h] of width 2d (Sec. 4.3).  All fp32. */
+typedef struct {
+  const float* w1;      /* device [r, 2d] */
+  const float* b1;      /* device [r] */
+  const float* w2;      /* device [L-2, r] */
+  const float* b2;      /* device [L-2] */
+  const float* prior;   /* device [L-2] normalised prior p~ (Eq. 2), or NULL */
+  float omega;          /* prior weight (ignored when prior == NULL) */
+} buddy_dm_weights;
+
+/* Per-layer KV caches and per-sequence positions (Eq. 9).
+ * Element (sequence i, kv head g, position p, channel e) of layer l's K cache
+ * is at  k_cache[l] + ((seq_off[i] * n_kv + g * cap[i] + p) * head_dim + e)
+ * elements (same for V): each sequence owns a head-major block of cap[i]
+ * positions; blocks must not overlap.  len[i] = cached positions n_i (equal
+ * for every layer).  pool_sum[i] = running fp32 sum over the cached positions
+ * of the first layer's V (the KV-aware planner's context, Sec. 4.3). */
+typedef struct {
+  void* const* k_cache;     /* host array [L] of device pointers (config dtype) */
+  void* const* v_cache;     /* host array [L] of device pointers */
+  const int64_t* seq_off;   /* device [batch] */
+  const int32_t* cap;       /* device [batch] */
+  int32_t* len;             /* device [batch] */
+  float* pool_sum;          /* device [batch, n_kv * hd] */
+  int32_t batch;            /* number of sequences the state holds */
+} buddy_kv_state;
+
+/* Creates a context on the current device; allocates its scratch. */
+BUDDY_API int buddy_create(const buddy_config* cfg, buddy_ctx** out);
+BUDDY_API void buddy_destroy(buddy_ctx* ctx);
+
+/* Registers the model: layers[0..L-1] and the Decision Module.  Pointers are
+ * retained.  Builds the TMA tensor descriptors of the bf16 weight matrices. */
+BUDDY_API int buddy_set_weights(buddy_ctx* ctx, const buddy_layer_weights* layers, const buddy_dm_weights* dm);
+
+/* Prefill / bulk append of n_new positions to layer `layer` for n_seq
+ * sequences (KV cache update, Eq. 9).  k_new, v_new: device
+ * [n_seq, n_new, n_kv, hd] (config dtype), written at positions
+ * len[s] .. len[s] + n_new - 1 of sequence s = seq_ids[j].  For layer 0 the
+ * pooled context pool_sum[s] is recomputed as the full sum over positions
+ * 0 .. len[s] + n_new - 1.  advance != 0 adds n_new to len[s] afterwards
+ * (pass it on the last layer appended).  seq_ids must be distinct.
+ * Device-checked: s < kv->batch,
+ * len[s] + n_new <= cap[s] and <= max_pos. */
+BUDDY_API int buddy_kv_append(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t layer, int32_t n_seq,
+                    const int32_t* seq_ids, int32_t n_new, const void* k_new, const void* v_new,
+                    int32_t advance, void* stream);
+
+/* The router alone (KV-aware planner + Decision Module + top-k, Sec. 4.2-4.3):
+ * for i < batch, pool = pool_sum[i] / len[i] (the cache must already hold the
+ * newest token at position len[i]-1), x = [pool expanded; h1[i]],
+ * s' as in buddy_dm_weights, selection = the k[i] largest s' (ties to the lower
+ * index).  h1: device [batch, d] fp32; k: device [batch] int32 in [1, L-2].
+ * Outputs (device, any may be NULL): sel_out [batch, L-2] int32 — executed
+ * layer ids (1..L-2, ascending) then -1; mask_out [batch, L] uint8 (first and
+ * last layer set); scores_out [batch, L-2] fp32. */
+BUDDY_API int buddy_route(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t batch, const float* h1,
+                const int32_t* k, int32_t* sel_out, uint8_t* mask_out, float* scores_out,
+                void* stream);
+
+/* One budget-routed decode step for sequences 0..batch-1 of `kv`.
+ * h_in: device [batch, d] fp32 (input of the first block); k: device [batch]
+ * int32 budgets in [1, L-2]; h_out: device [batch, d] fp32, the hidden state
+ * after the last block (must not alias h_in).  Optional device outputs (NULL
+ * to skip): mask_out [batch, L] uint8; rows_out [L, batch] int32 (for layer l
+ * the ascending ids of the sequences that execute it, then unspecified);
+ * count_out [L] int32 (their number); scores_out [batch, L-2] fp32.
+ * Every layer's cache receives one position per sequence (zeros for skipped
+ * layers) and len[i] += 1.  Device-checked: k[i] in range, len[i] + 1 <= cap[i]
+ * and <= max_pos; on failure nothing is written. */
+BUDDY_API int buddy_decode_step(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t batch, const float* h_in,
+                      const int32_t* k, float* h_out, uint8_t* mask_out, int32_t* rows_out,
+                      int32_t* count_out, float* scores_out, void* stream);
+
+/* buddy_decode_step with HOST buffers: h_in_host [batch, d] fp32, k_host
+ * [batch] int32, h_out_host [batch, d] fp32, mask_host [batch, L] uint8 (or
+ * NULL).  Copies the inputs to device staging buffers, runs the step, copies
+ * the outputs back and synchronises the stream before returning.  Pinned host
+ * memory gives asynchronous copies; pageable memory works but is slower. */
+BUDDY_API int buddy_decode_step_host(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t batch,
+                           const float* h_in_host, const int32_t* k_host, float* h_out_host,
+                           uint8_t* mask_host, void* stream);
+
+/* Execution options.  use_graph != 0: buddy_decode_step replays a CUDA graph
+ * captured per (batch, kv state, stream) on first use, with a device-set
+ * conditional node per layer so that layers no sequence selected cost no
+ * kernel launches.  The graph bakes in the pointers of that call; a call with
+ * other pointers re-captures. */
+BUDDY_API int buddy_set_options(buddy_ctx* ctx, int32_t use_graph);
+
+/* Kernel classes reported by the profiler. */
+enum {
+  BUDDY_PROF_CHECK = 0, BUDDY_PROF_RMSNORM, BUDDY_PROF_GEMM_QKV, BUDDY_PROF_QKV_FINALIZE,
+  BUDDY_PROF_ATTENTION, BUDDY_PROF_GEMM_O, BUDDY_PROF_GEMM_GATE_UP, BUDDY_PROF_GEMM_DOWN,
+  BUDDY_PROF_ROUTE, BUDDY_PROF_COMPACT, BUDDY_PROF_OTHER, BUDDY_PROF_NCLASS
+};
+
+/* Per-kernel-class timing.  With on != 0, direct-launch decode steps
+ * (use_graph == 0) record a CUDA event pair on the launching stream around
+ * every kernel launch, and count the launches.  buddy_profile_read
+ * synchronises those events, writes per class the summed milliseconds and the
+ * launch count (arrays of n_cls entries, n_cls <= BUDDY_PROF_NCLASS), and
+ * clears the records.  buddy_profile_class_name gives a class's name. */
+BUDDY_API int buddy_set_profiling(buddy_ctx* ctx, int32_t on);
+BUDDY_API int buddy_profile_read(buddy_ctx* ctx, int32_t n_cls, float* ms, int32_t* launches);
+BUDDY_API const char* buddy_profile_class_name(int32_t cls);
+
+/* Synchronises `stream`, stores the device error flag bits (BUDDY_DEV_*) in
+ * *flags and clears them.  Returns BUDDY_ERR_DEVICE if any bit was set. */
+BUDDY_API int buddy_device_status(buddy_ctx* ctx, void* stream, int32_t* flags);
+
+/* Budget b in (0, 1] to middle-layer count: k = round(b * L) - 2 (Eq. 2,
+ * ties to even), clamped to the action space [1, L-2] (Sec. 4.4).
+ * Returns -1 if n_layers < 3 or b is not finite. */
+BUDDY_API int32_t buddy_budget_to_k(float b, int32_t n_layers);
+
+BUDDY_API const char* buddy_error_string(int32_t code);
+BUDDY_API int32_t buddy_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BUDDY_H_ */

@@ -61,16 +61,17 @@ def build_model(shape: ModelShape, seed: int, *, layer_source=None, dm_source=No
 
 def build_state(shape: ModelShape, seed: int, n_ctx: Sequence[int],
                 layers: Optional[Sequence[int]] = None,
-                seqs: Optional[Sequence[int]] = None) -> O.KVState:
-    """Prefilled caches (positions 0..n_i-1) for the given layers and sequences."""
+                seqs: Optional[Sequence[int]] = None, gen_device: str = "cpu") -> O.KVState:
+    """Prefilled caches (positions 0..n_i-1) for the given layers and sequences.
+    `gen_device` only chooses where the generator runs (values are identical)."""
     st = O.KVState(n_ctx)
     layers = range(shape.n_layers) if layers is None else layers
     seqs = range(len(n_ctx)) if seqs is None else seqs
     for l in layers:
         for i in seqs:
             n = int(n_ctx[i])
-            K = to_f64(synth.kv_block(shape, seed, "k", l, i, 0, n))
-            V = to_f64(synth.kv_block(shape, seed, "v", l, i, 0, n))
+            K = to_f64(synth.kv_block(shape, seed, "k", l, i, 0, n, gen_device))
+            V = to_f64(synth.kv_block(shape, seed, "v", l, i, 0, n, gen_device))
             st.set(l, i, K, V)
     return st
 

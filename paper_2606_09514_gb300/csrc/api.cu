@@ -1,0 +1,532 @@
+// C-ABI of libbuddy: argument validation, scratch management, and the
+// orchestration of one budget-routed decode step (direct launches or a CUDA
+// graph whose middle layers sit behind device-set conditional nodes).
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <functional>
+#include <new>
+#include <tuple>
+
+#include "../../include/buddy.h"
+#include "internal.h"
+
+using namespace buddy;
+
+struct buddy_ctx {
+  Ctx c;
+  cudaStream_t cap_stream = nullptr;   // graph capture (the legacy stream cannot be captured)
+  cudaStream_t body_stream = nullptr;  // capture of conditional bodies
+};
+
+#define CK(x)                                                     \
+  do {                                                            \
+    cudaError_t e_ = (x);                                         \
+    if (e_ != cudaSuccess) {                                      \
+      fprintf(stderr, "libbuddy: %s -> %s (%s:%d)\n", #x,         \
+              cudaGetErrorString(e_), __FILE__, __LINE__);        \
+      return BUDDY_ERR_CUDA;                                      \
+    }                                                             \
+  } while (0)
+
+namespace buddy {
+bool Ctx::GraphKey::operator<(const GraphKey& o) const {
+  return std::tie(B, h_in, k, h_out, mask, rows, count, scores, stream, kvp) <
+         std::tie(o.B, o.h_in, o.k, o.h_out, o.mask, o.rows, o.count, o.scores, o.stream, o.kvp);
+}
+int gemm_tc_prepare(Ctx& c);   // gemm_tc.cu
+}  // namespace buddy
+
+template <typename T>
+static cudaError_t dalloc(T** p, size_t n) {
+  *p = nullptr;
+  if (n == 0) n = 1;
+  return cudaMalloc((void**)p, n * sizeof(T));
+}
+
+static void free_ctx(buddy_ctx* x) {
+  if (!x) return;
+  Ctx& c = x->c;
+  for (auto& kv : c.graphs) cudaGraphExecDestroy(kv.second);
+  for (cudaEvent_t e : c.ev_pool) cudaEventDestroy(e);
+  void* ptrs[] = {c.rope_cos, c.rope_sin, c.status, c.xn, c.act, c.attn_out, c.qkv, c.q,
+                  c.attn_m, c.attn_l, c.attn_acc, c.dm_u, c.mask, c.sel, c.scores, c.rows,
+                  c.count, c.h_in_stage, c.h_out_stage, c.k_stage, c.mask_stage, c.tmaps,
+                  c.gemm_ws, c.gemm_ctr};
+  for (void* p : ptrs)
+    if (p) cudaFree(p);
+  if (x->cap_stream) cudaStreamDestroy(x->cap_stream);
+  if (x->body_stream) cudaStreamDestroy(x->body_stream);
+  delete x;
+}
+
+extern "C" int32_t buddy_version(void) { return 1; }
+
+extern "C" const char* buddy_error_string(int32_t code) {
+  switch (code) {
+    case BUDDY_OK: return "ok";
+    case BUDDY_ERR_ARG: return "invalid argument";
+    case BUDDY_ERR_RANGE: return "value out of range";
+    case BUDDY_ERR_CUDA: return "CUDA runtime error";
+    case BUDDY_ERR_DEVICE: return "device error flag raised";
+    case BUDDY_ERR_STATE: return "invalid call order (weights not set?)";
+    default: return "unknown error";
+  }
+}
+
+extern "C" int32_t buddy_budget_to_k(float b, int32_t n_layers) {
+  if (n_layers < 3 || !std::isfinite(b)) return -1;
+  // k = round(b L) - 2 with ties to even (Eq. 2), clamped to {1..L-2} (Sec. 4.4)
+  const double k = std::nearbyint((double)b * (double)n_layers) - 2.0;
+  const double lo = 1.0, hi = (double)(n_layers - 2);
+  return (int32_t)(k < lo ? lo : (k > hi ? hi : k));
+}
+
+extern "C" int buddy_create(const buddy_config* cfg, buddy_ctx** out) {
+  if (!cfg || !out) return BUDDY_ERR_ARG;
+  *out = nullptr;
+  const buddy_config& g = *cfg;
+  if (g.n_layers < 3 || g.n_layers > kMaxLayers || g.d_model <= 0 || g.n_q_heads <= 0 ||
+      g.n_kv_heads <= 0 || (g.head_dim != 64 && g.head_dim != 128) ||
+      g.n_q_heads % g.n_kv_heads != 0 || g.n_q_heads / g.n_kv_heads > 8 ||
+      g.d_model != g.n_q_heads * g.head_dim || g.d_model % 64 != 0 || g.ffn_dim <= 0 ||
+      g.ffn_dim % 8 != 0 || g.dm_hidden <= 0 || g.max_batch < 1 || g.max_batch > kMaxBatch ||
+      g.max_pos < 1 || (g.dtype != BUDDY_DTYPE_F32 && g.dtype != BUDDY_DTYPE_BF16) ||
+      !(g.rms_eps > 0.f) || !(g.rope_theta > 0.f))
+    return BUDDY_ERR_ARG;
+  buddy_ctx* x = new (std::nothrow) buddy_ctx();
+  if (!x) return BUDDY_ERR_CUDA;
+  Ctx& c = x->c;
+  c.cfg = g;
+  c.L = g.n_layers; c.Lm = g.n_layers - 2; c.d = g.d_model; c.nq = g.n_q_heads;
+  c.nkv = g.n_kv_heads; c.hd = g.head_dim; c.F = g.ffn_dim; c.r = g.dm_hidden;
+  c.qd = c.nq * c.hd; c.kvd = c.nkv * c.hd; c.qkvN = c.qd + 2 * c.kvd;
+  c.maxB = g.max_batch; c.max_pos = g.max_pos; c.dtype = g.dtype;
+  c.esz = g.dtype == BUDDY_DTYPE_BF16 ? 2 : 4;
+  auto fail = [&](cudaError_t e) {
+    fprintf(stderr, "libbuddy: create: %s\n", cudaGetErrorString(e));
+    free_ctx(x);
+    return BUDDY_ERR_CUDA;
+  };
+  cudaError_t e;
+  if ((e = cudaGetDevice(&c.device)) != cudaSuccess) return fail(e);
+  if ((e = cudaDeviceGetAttribute(&c.num_sms, cudaDevAttrMultiProcessorCount, c.device)) != cudaSuccess)
+    return fail(e);
+  const size_t B = c.maxB;
+  c.attn_chunk = 128;
+  c.attn_max_chunks = (c.max_pos + c.attn_chunk - 1) / c.attn_chunk;
+  const size_t hmax = (size_t)c.max_pos * (c.hd / 2);
+  if ((e = dalloc(&c.rope_cos, hmax)) || (e = dalloc(&c.rope_sin, hmax)) ||
+      (e = dalloc(&c.status, 4)) ||
+      (e = cudaMalloc(&c.xn, B * c.d * c.esz)) || (e = cudaMalloc(&c.act, B * c.F * c.esz)) ||
+      (e = cudaMalloc(&c.attn_out, B * c.qd * c.esz)) || (e = dalloc(&c.qkv, B * c.qkvN)) ||
+      (e = dalloc(&c.q, B * c.qd)) ||
+      (e = dalloc(&c.attn_m, B * c.nq * c.attn_max_chunks)) ||
+      (e = dalloc(&c.attn_l, B * c.nq * c.attn_max_chunks)) ||
+      (e = dalloc(&c.attn_acc, B * c.nq * c.attn_max_chunks * c.hd)) ||
+      (e = dalloc(&c.dm_u, B * c.r)) || (e = dalloc(&c.mask, B * c.L)) ||
+      (e = dalloc(&c.sel, B * c.Lm)) || (e = dalloc(&c.scores, B * c.Lm)) ||
+      (e = dalloc(&c.rows, (size_t)c.L * B)) || (e = dalloc(&c.count, (size_t)c.L)) ||
+      (e = dalloc(&c.h_in_stage, B * c.d)) || (e = dalloc(&c.h_out_stage, B * c.d)) ||
+      (e = dalloc(&c.k_stage, B)) || (e = dalloc(&c.mask_stage, B * c.L)))
+    return fail(e);
+  if ((e = cudaMemset(c.status, 0, 4 * sizeof(int32_t))) != cudaSuccess) return fail(e);
+  if ((e = cudaStreamCreateWithFlags(&x->cap_stream, cudaStreamNonBlocking)) != cudaSuccess ||
+      (e = cudaStreamCreateWithFlags(&x->body_stream, cudaStreamNonBlocking)) != cudaSuccess)
+    return fail(e);
+  launch_rope_table(c.rope_cos, c.rope_sin, c.max_pos, c.hd, (double)g.rope_theta, x->cap_stream);
+  if ((e = cudaGetLastError()) != cudaSuccess || (e = cudaStreamSynchronize(x->cap_stream)) != cudaSuccess)
+    return fail(e);
+  *out = x;
+  return BUDDY_OK;
+}
+
+extern "C" void buddy_destroy(buddy_ctx* ctx) {
+  if (!ctx) return;
+  cudaDeviceSynchronize();
+  free_ctx(ctx);
+}
+
+extern "C" int buddy_set_weights(buddy_ctx* ctx, const buddy_layer_weights* layers,
+                                 const buddy_dm_weights* dm) {
+  if (!ctx || !layers || !dm) return BUDDY_ERR_ARG;
+  Ctx& c = ctx->c;
+  for (int l = 0; l < c.L; ++l) {
+    const buddy_layer_weights& w = layers[l];
+    if (!w.attn_norm || !w.w_qkv || !w.w_o || !w.ffn_norm || !w.w_gate_up || !w.w_down)
+      return BUDDY_ERR_ARG;
+    if (c.cfg.qkv_bias && !w.b_qkv) return BUDDY_ERR_ARG;
+  }
+  if (!dm->w1 || !dm->b1 || !dm->w2 || !dm->b2) return BUDDY_ERR_ARG;
+  c.layers.assign(layers, layers + c.L);
+  if (!c.cfg.qkv_bias)
+    for (auto& w : c.layers) w.b_qkv = nullptr;
+  c.dm = *dm;
+  for (auto& kv : c.graphs) cudaGraphExecDestroy(kv.second);
+  c.graphs.clear();
+  c.have_weights = true;
+  const int rc = gemm_tc_prepare(c);
+  if (rc != BUDDY_OK) {
+    c.have_weights = false;
+    return rc;
+  }
+  return BUDDY_OK;
+}
+
+extern "C" int buddy_set_options(buddy_ctx* ctx, int32_t use_graph) {
+  if (!ctx) return BUDDY_ERR_ARG;
+  ctx->c.use_graph = use_graph ? 1 : 0;
+  return BUDDY_OK;
+}
+
+static int check_kv(const Ctx& c, const buddy_kv_state* kv, int need_batch) {
+  if (!kv || !kv->k_cache || !kv->v_cache || !kv->seq_off || !kv->cap || !kv->len || !kv->pool_sum)
+    return BUDDY_ERR_ARG;
+  if (kv->batch < need_batch || kv->batch < 1) return BUDDY_ERR_ARG;
+  for (int l = 0; l < c.L; ++l)
+    if (!kv->k_cache[l] || !kv->v_cache[l]) return BUDDY_ERR_ARG;
+  return BUDDY_OK;
+}
+
+extern "C" int buddy_device_status(buddy_ctx* ctx, void* stream, int32_t* flags) {
+  if (!ctx || !flags) return BUDDY_ERR_ARG;
+  Ctx& c = ctx->c;
+  cudaStream_t s = (cudaStream_t)stream;
+  int32_t h[2] = {0, 0};
+  CK(cudaMemcpyAsync(h, c.status, 2 * sizeof(int32_t), cudaMemcpyDeviceToHost, s));
+  CK(cudaStreamSynchronize(s));
+  CK(cudaMemsetAsync(c.status, 0, 2 * sizeof(int32_t), s));
+  CK(cudaStreamSynchronize(s));
+  *flags = h[0];
+  return h[0] ? BUDDY_ERR_DEVICE : BUDDY_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Profiler: an event pair around each launch group (direct-launch mode only).
+// ---------------------------------------------------------------------------
+static cudaEvent_t take_event(Ctx& c) {
+  if (c.ev_used == c.ev_pool.size()) {
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    c.ev_pool.push_back(e);
+  }
+  return c.ev_pool[c.ev_used++];
+}
+
+struct ProfScope {
+  Ctx& c;
+  cudaStream_t s;
+  Ctx::ProfRec rec{};
+  bool on;
+  ProfScope(Ctx& c_, cudaStream_t s_, int cls, int launches, bool on_) : c(c_), s(s_), on(on_) {
+    if (!on) return;
+    rec.cls = cls;
+    rec.launches = launches;
+    rec.a = take_event(c);
+    rec.b = take_event(c);
+    on = rec.a && rec.b;
+    if (on) cudaEventRecord(rec.a, s);
+  }
+  ~ProfScope() {
+    if (!on) return;
+    cudaEventRecord(rec.b, s);
+    c.prof.push_back(rec);
+  }
+};
+
+extern "C" int buddy_set_profiling(buddy_ctx* ctx, int32_t on) {
+  if (!ctx) return BUDDY_ERR_ARG;
+  ctx->c.profiling = on ? 1 : 0;
+  return BUDDY_OK;
+}
+
+extern "C" const char* buddy_profile_class_name(int32_t cls) {
+  static const char* names[BUDDY_PROF_NCLASS] = {"check", "rmsnorm", "gemm_qkv", "qkv_finalize",
+                                                 "attention", "gemm_o", "gemm_gate_up", "gemm_down",
+                                                 "route", "compact", "other"};
+  return (cls >= 0 && cls < BUDDY_PROF_NCLASS) ? names[cls] : "unknown";
+}
+
+extern "C" int buddy_profile_read(buddy_ctx* ctx, int32_t n_cls, float* ms, int32_t* launches) {
+  if (!ctx || n_cls < 0 || n_cls > BUDDY_PROF_NCLASS || (n_cls > 0 && (!ms || !launches)))
+    return BUDDY_ERR_ARG;
+  Ctx& c = ctx->c;
+  for (int i = 0; i < n_cls; ++i) {
+    ms[i] = 0.f;
+    launches[i] = 0;
+  }
+  for (const auto& r : c.prof) {
+    CK(cudaEventSynchronize(r.b));
+    float t = 0.f;
+    CK(cudaEventElapsedTime(&t, r.a, r.b));
+    if (r.cls < n_cls) {
+      ms[r.cls] += t;
+      launches[r.cls] += r.launches;
+    }
+  }
+  c.prof.clear();
+  c.ev_used = 0;
+  return BUDDY_OK;
+}
+
+// ---------------------------------------------------------------------------
+// GEMM dispatch
+// ---------------------------------------------------------------------------
+static void run_gemm(const Ctx& c, int epi, GemmArgs a, int layer, int which, cudaStream_t s) {
+  a.status = c.status;
+  if (c.use_tc) {
+    a.tmap_w = c.tmaps + (size_t)layer * 4 + which;
+    launch_gemm_tc(c, epi, a, s);
+  } else {
+    launch_gemm_simt(c, epi, a, s);
+  }
+}
+
+// One decoder block on the rows of `sel` (Eq. 1 executed branch): the residual
+// stream H is updated in place for those rows; for layer 0 the input comes
+// from `src` and the output goes to `H`.
+static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, const float* src,
+                          float* H, cudaStream_t s, bool prof) {
+  const buddy_layer_weights& W = c.layers[l];
+  {
+    ProfScope p(c, s, BUDDY_PROF_RMSNORM, 1, prof);
+    launch_rmsnorm(c, src, sel, W.attn_norm, c.xn, s);
+  }
+  GemmArgs g{};
+  g.sel = sel;
+  g.max_m = sel.n;
+  g.W = W.w_qkv; g.X = c.xn; g.N = c.qkvN; g.K = c.d; g.out_f32 = c.qkv;
+  {
+    ProfScope p(c, s, BUDDY_PROF_GEMM_QKV, 1, prof);
+    run_gemm(c, EPI_STORE_F32, g, l, 0, s);
+  }
+  {
+    ProfScope p(c, s, BUDDY_PROF_QKV_FINALIZE, 1, prof);
+    launch_qkv_finalize(c, c.qkv, W.b_qkv, sel, kv, l, c.q, l == 0 ? kv.pool_sum : nullptr, s);
+  }
+  {
+    ProfScope p(c, s, BUDDY_PROF_ATTENTION, 2, prof);
+    launch_attention(c, sel, kv, l, c.q, c.attn_out, s);
+  }
+  g = GemmArgs{};
+  g.sel = sel; g.max_m = sel.n;
+  g.W = W.w_o; g.X = c.attn_out; g.N = c.d; g.K = c.qd; g.resid_src = src; g.resid_dst = H;
+  {
+    ProfScope p(c, s, BUDDY_PROF_GEMM_O, 1, prof);
+    run_gemm(c, EPI_RESID, g, l, 1, s);
+  }
+  {
+    ProfScope p(c, s, BUDDY_PROF_RMSNORM, 1, prof);
+    launch_rmsnorm(c, H, sel, W.ffn_norm, c.xn, s);
+  }
+  g = GemmArgs{};
+  g.sel = sel; g.max_m = sel.n;
+  g.W = W.w_gate_up; g.X = c.xn; g.N = c.F; g.K = c.d; g.out_act = c.act;
+  {
+    ProfScope p(c, s, BUDDY_PROF_GEMM_GATE_UP, 1, prof);
+    run_gemm(c, EPI_SWIGLU, g, l, 2, s);
+  }
+  g = GemmArgs{};
+  g.sel = sel; g.max_m = sel.n;
+  g.W = W.w_down; g.X = c.act; g.N = c.d; g.K = c.F; g.resid_src = H; g.resid_dst = H;
+  {
+    ProfScope p(c, s, BUDDY_PROF_GEMM_DOWN, 1, prof);
+    run_gemm(c, EPI_RESID, g, l, 3, s);
+  }
+}
+
+struct StepIO {
+  int B;
+  const float* h_in;
+  const int32_t* k;
+  float* h_out;
+  uint8_t* mask_out;
+  int32_t* rows_out;
+  int32_t* count_out;
+  float* scores_out;
+};
+
+// Enqueues the whole step.  When `body_stream` is non-null the caller is
+// capturing `s` into a graph: each middle layer becomes a conditional node
+// whose body runs iff count[l] > 0.
+static int enqueue_step(buddy_ctx* x, const buddy_kv_state& kv, const StepIO& io, cudaStream_t s,
+                        bool capture) {
+  Ctx& c = x->c;
+  const int B = io.B;
+  const bool prof = c.profiling && !capture;
+  {
+    ProfScope p(c, s, BUDDY_PROF_CHECK, 1, prof);
+    launch_step_check(c, B, io.k, kv.len, kv.cap, 1, c.status, s);
+  }
+  const RowSel all{nullptr, nullptr, B};
+  enqueue_layer(c, kv, 0, all, io.h_in, io.h_out, s, prof);
+  {
+    ProfScope p(c, s, BUDDY_PROF_ROUTE, 2, prof);
+    launch_route(c, B, io.h_out, kv.pool_sum, kv.len, 1, io.k, c.mask, c.sel, c.scores, s);
+  }
+  {
+    ProfScope p(c, s, BUDDY_PROF_COMPACT, 1, prof);
+    launch_compact(c, B, c.mask, kv, c.rows, c.count, s);
+  }
+  int32_t hcount[kMaxLayers];
+  if (prof) {
+    // profiling: launch only the layers some sequence selected
+    CK(cudaMemcpyAsync(hcount, c.count, sizeof(int32_t) * c.L, cudaMemcpyDeviceToHost, s));
+    CK(cudaStreamSynchronize(s));
+  }
+  for (int l = 1; l < c.L - 1; ++l) {
+    const RowSel sel{c.rows + (size_t)l * B, c.count + l, B};
+    if (!capture) {
+      if (!prof || hcount[l] > 0) enqueue_layer(c, kv, l, sel, io.h_out, io.h_out, s, prof);
+      continue;
+    }
+    cudaGraph_t g = nullptr;
+    cudaStreamCaptureStatus st;
+    CK(cudaStreamGetCaptureInfo(s, &st, nullptr, &g, nullptr, nullptr, nullptr));
+    cudaGraphConditionalHandle h;
+    CK(cudaGraphConditionalHandleCreate(&h, g, 0, cudaGraphCondAssignDefault));
+    launch_set_conditional(h, c.count + l, c.status, s);
+    const cudaGraphNode_t* deps = nullptr;
+    const cudaGraphEdgeData* edata = nullptr;
+    size_t ndeps = 0;
+    CK(cudaStreamGetCaptureInfo(s, &st, nullptr, &g, &deps, &edata, &ndeps));
+    cudaGraphNodeParams p{};
+    p.type = cudaGraphNodeTypeConditional;
+    p.conditional.handle = h;
+    p.conditional.type = cudaGraphCondTypeIf;
+    p.conditional.size = 1;
+    cudaGraphNode_t node;
+    CK(cudaGraphAddNode(&node, g, deps, edata, ndeps, &p));
+    cudaGraph_t body = p.conditional.phGraph_out[0];
+    CK(cudaStreamUpdateCaptureDependencies(s, &node, nullptr, 1, cudaStreamSetCaptureDependencies));
+    CK(cudaStreamBeginCaptureToGraph(x->body_stream, body, nullptr, nullptr, 0,
+                                     cudaStreamCaptureModeRelaxed));
+    enqueue_layer(c, kv, l, sel, io.h_out, io.h_out, x->body_stream, false);
+    cudaGraph_t done = nullptr;
+    CK(cudaStreamEndCapture(x->body_stream, &done));
+  }
+  enqueue_layer(c, kv, c.L - 1, all, io.h_out, io.h_out, s, prof);
+  {
+    ProfScope p(c, s, BUDDY_PROF_OTHER, 1, prof);
+    launch_advance(c, B, kv.len, 1, nullptr, s);
+  }
+  if (io.mask_out) CK(cudaMemcpyAsync(io.mask_out, c.mask, (size_t)B * c.L, cudaMemcpyDeviceToDevice, s));
+  if (io.rows_out)
+    CK(cudaMemcpyAsync(io.rows_out, c.rows, (size_t)B * c.L * sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
+  if (io.count_out)
+    CK(cudaMemcpyAsync(io.count_out, c.count, (size_t)c.L * sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
+  if (io.scores_out)
+    CK(cudaMemcpyAsync(io.scores_out, c.scores, (size_t)B * c.Lm * sizeof(float), cudaMemcpyDeviceToDevice, s));
+  CK(cudaGetLastError());
+  return BUDDY_OK;
+}
+
+static int run_step(buddy_ctx* x, const buddy_kv_state* kv, const StepIO& io, cudaStream_t s) {
+  Ctx& c = x->c;
+  if (!c.use_graph) return enqueue_step(x, *kv, io, s, false);
+  Ctx::GraphKey key{io.B, io.h_in, io.k, io.h_out, io.mask_out, io.rows_out, io.count_out,
+                    io.scores_out, s, {}};
+  for (int l = 0; l < c.L; ++l) {
+    key.kvp.push_back(kv->k_cache[l]);
+    key.kvp.push_back(kv->v_cache[l]);
+  }
+  key.kvp.push_back(kv->seq_off);
+  key.kvp.push_back(kv->cap);
+  key.kvp.push_back(kv->len);
+  key.kvp.push_back(kv->pool_sum);
+  auto it = c.graphs.find(key);
+  if (it == c.graphs.end()) {
+    cudaStream_t cs = x->cap_stream;
+    CK(cudaStreamBeginCapture(cs, cudaStreamCaptureModeRelaxed));
+    int rc = enqueue_step(x, *kv, io, cs, true);
+    cudaGraph_t g = nullptr;
+    cudaError_t e = cudaStreamEndCapture(cs, &g);
+    if (rc != BUDDY_OK) {
+      if (g) cudaGraphDestroy(g);
+      return rc;
+    }
+    CK(e);
+    cudaGraphExec_t ge = nullptr;
+    e = cudaGraphInstantiate(&ge, g, 0);
+    cudaGraphDestroy(g);
+    CK(e);
+    it = c.graphs.emplace(key, ge).first;
+  }
+  CK(cudaGraphLaunch(it->second, s));
+  return BUDDY_OK;
+}
+
+extern "C" int buddy_decode_step(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t batch,
+                                 const float* h_in, const int32_t* k, float* h_out,
+                                 uint8_t* mask_out, int32_t* rows_out, int32_t* count_out,
+                                 float* scores_out, void* stream) {
+  if (!ctx) return BUDDY_ERR_ARG;
+  Ctx& c = ctx->c;
+  if (!c.have_weights) return BUDDY_ERR_STATE;
+  if (batch < 1 || batch > c.maxB || !h_in || !k || !h_out || h_in == h_out) return BUDDY_ERR_ARG;
+  int rc = check_kv(c, kv, batch);
+  if (rc) return rc;
+  StepIO io{batch, h_in, k, h_out, mask_out, rows_out, count_out, scores_out};
+  return run_step(ctx, kv, io, (cudaStream_t)stream);
+}
+
+extern "C" int buddy_decode_step_host(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t batch,
+                                      const float* h_in_host, const int32_t* k_host,
+                                      float* h_out_host, uint8_t* mask_host, void* stream) {
+  if (!ctx) return BUDDY_ERR_ARG;
+  Ctx& c = ctx->c;
+  if (!c.have_weights) return BUDDY_ERR_STATE;
+  if (batch < 1 || batch > c.maxB || !h_in_host || !k_host || !h_out_host) return BUDDY_ERR_ARG;
+  int rc = check_kv(c, kv, batch);
+  if (rc) return rc;
+  cudaStream_t s = (cudaStream_t)stream;
+  CK(cudaMemcpyAsync(c.h_in_stage, h_in_host, (size_t)batch * c.d * sizeof(float), cudaMemcpyHostToDevice, s));
+  CK(cudaMemcpyAsync(c.k_stage, k_host, (size_t)batch * sizeof(int32_t), cudaMemcpyHostToDevice, s));
+  StepIO io{batch, c.h_in_stage, c.k_stage, c.h_out_stage, mask_host ? c.mask_stage : nullptr,
+            nullptr, nullptr, nullptr};
+  rc = run_step(ctx, kv, io, s);
+  if (rc) return rc;
+  CK(cudaMemcpyAsync(h_out_host, c.h_out_stage, (size_t)batch * c.d * sizeof(float), cudaMemcpyDeviceToHost, s));
+  if (mask_host) CK(cudaMemcpyAsync(mask_host, c.mask_stage, (size_t)batch * c.L, cudaMemcpyDeviceToHost, s));
+  CK(cudaStreamSynchronize(s));
+  return BUDDY_OK;
+}
+
+extern "C" int buddy_route(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t batch, const float* h1,
+                           const int32_t* k, int32_t* sel_out, uint8_t* mask_out, float* scores_out,
+                           void* stream) {
+  if (!ctx) return BUDDY_ERR_ARG;
+  Ctx& c = ctx->c;
+  if (!c.have_weights) return BUDDY_ERR_STATE;
+  if (batch < 1 || batch > c.maxB || !h1 || !k) return BUDDY_ERR_ARG;
+  if (!kv || !kv->len || !kv->pool_sum || !kv->cap || kv->batch < batch) return BUDDY_ERR_ARG;
+  cudaStream_t s = (cudaStream_t)stream;
+  // positions: the cache already holds the newest token (len >= 1)
+  launch_step_check(c, batch, k, kv->len, kv->cap, 0, c.status, s);
+  launch_route(c, batch, h1, kv->pool_sum, kv->len, 0, k, mask_out, sel_out, scores_out, s);
+  CK(cudaGetLastError());
+  return BUDDY_OK;
+}
+
+extern "C" int buddy_kv_append(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t layer,
+                               int32_t n_seq, const int32_t* seq_ids, int32_t n_new,
+                               const void* k_new, const void* v_new, int32_t advance, void* stream) {
+  if (!ctx) return BUDDY_ERR_ARG;
+  Ctx& c = ctx->c;
+  if (layer < 0 || layer >= c.L || n_seq < 1 || n_seq > kMaxBatch * 64 || n_new < 0 || !seq_ids)
+    return BUDDY_ERR_ARG;
+  if (n_new > 0 && (!k_new || !v_new)) return BUDDY_ERR_ARG;
+  if (n_new > 65535) return BUDDY_ERR_RANGE;
+  int rc = check_kv(c, kv, 1);
+  if (rc) return rc;
+  cudaStream_t s = (cudaStream_t)stream;
+  launch_kv_check(c, n_seq, seq_ids, n_new, kv->batch, kv->len, kv->cap, c.status, s);
+  if (n_new > 0) launch_kv_append(c, *kv, layer, n_seq, seq_ids, n_new, k_new, v_new, s);
+  if (layer == 0) launch_pool_refresh(c, *kv, n_seq, seq_ids, n_new, s);
+  if (advance && n_new > 0) launch_advance(c, n_seq, kv->len, n_new, seq_ids, s);
+  CK(cudaGetLastError());
+  return BUDDY_OK;
+}

@@ -1,0 +1,151 @@
+// Host-side internals of libbuddy: context layout and kernel launchers.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <map>
+#include <vector>
+
+#include "../../include/buddy.h"
+
+namespace buddy {
+
+constexpr int kMaxLayers = 128;
+constexpr int kMaxBatch = 1024;
+
+// Per-layer K/V base pointers passed by value to kernels that touch many layers.
+struct LayerPtrs {
+  void* k[kMaxLayers];
+  void* v[kMaxLayers];
+};
+
+// Where the row list of a layer comes from: identity (rows == nullptr) with a
+// fixed count, or a device list with a device count.
+struct RowSel {
+  const int32_t* rows;    // device [max_batch] or nullptr (identity)
+  const int32_t* count;   // device scalar or nullptr (use n)
+  int n;                  // count when `count` is null; upper bound otherwise
+};
+
+enum GemmEpi { EPI_STORE_F32 = 0, EPI_RESID = 1, EPI_SWIGLU = 2 };
+
+struct GemmArgs {
+  const void* W;          // [N_rows, K] (weight dtype)
+  const void* X;          // [m, K] compact activations (act dtype)
+  int N;                  // output features (for SWIGLU: F, with W of 2F rows)
+  int K;
+  RowSel sel;             // m = row count; rows map j -> sequence for EPI_RESID
+  int max_m;              // grid sizing bound
+  // epilogues
+  float* out_f32;         // EPI_STORE_F32: [m, N]
+  void* out_act;          // EPI_SWIGLU: [m, N] act dtype
+  const float* resid_src; // EPI_RESID: dst[i] = src[i] + acc  (may equal dst)
+  float* resid_dst;
+  const int32_t* status;
+  // tcgen05 path: tensor maps (device-side copies live in the context)
+  const CUtensorMap* tmap_w;
+  const CUtensorMap* tmap_x;
+  int splits;             // split-K factor chosen by the host
+  float* ws;              // split-K partial workspace
+  int32_t* tile_ctr;      // split-K arrival counters (self-resetting)
+};
+
+struct Ctx;
+
+// Kernel launchers (kernels.cu)
+void launch_rope_table(float* cos_t, float* sin_t, int max_pos, int hd, double theta, cudaStream_t s);
+void launch_step_check(const Ctx& c, int B, const int32_t* k, const int32_t* len, const int32_t* cap,
+                       int extra_pos, int32_t* status, cudaStream_t s);
+void launch_kv_check(const Ctx& c, int n_seq, const int32_t* seq_ids, int n_new, int batch,
+                     const int32_t* len, const int32_t* cap, int32_t* status, cudaStream_t s);
+void launch_rmsnorm(const Ctx& c, const float* H, RowSel sel, const float* gamma, void* xn,
+                    cudaStream_t s);
+void launch_qkv_finalize(const Ctx& c, const float* qkv, const float* bias, RowSel sel,
+                         const buddy_kv_state& kv, int layer, float* q_out, float* pool,
+                         cudaStream_t s);
+void launch_attention(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q,
+                      void* attn_out, cudaStream_t s);
+void launch_route(const Ctx& c, int B, const float* h1, const float* pool, const int32_t* len,
+                  int len_bias, const int32_t* k, uint8_t* mask, int32_t* sel, float* scores,
+                  cudaStream_t s);
+void launch_compact(const Ctx& c, int B, const uint8_t* mask, const buddy_kv_state& kv,
+                    int32_t* rows, int32_t* count, cudaStream_t s);
+void launch_advance(const Ctx& c, int B, int32_t* len, int by, const int32_t* seq_ids, cudaStream_t s);
+void launch_kv_append(const Ctx& c, const buddy_kv_state& kv, int layer, int n_seq,
+                      const int32_t* seq_ids, int n_new, const void* k_new, const void* v_new,
+                      cudaStream_t s);
+void launch_pool_refresh(const Ctx& c, const buddy_kv_state& kv, int n_seq, const int32_t* seq_ids,
+                         int n_new, cudaStream_t s);
+void launch_set_conditional(cudaGraphConditionalHandle h, const int32_t* count, const int32_t* status,
+                            cudaStream_t s);
+
+// GEMMs (gemm_simt.cu, gemm_tc.cu)
+void launch_gemm_simt(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s);
+bool gemm_tc_supported(const Ctx& c);
+void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s);
+
+struct Ctx {
+  buddy_config cfg;
+  int L, Lm, d, nq, nkv, hd, F, r, qd, kvd, qkvN, maxB, max_pos;
+  int dtype;
+  size_t esz;
+  int device, num_sms;
+
+  bool have_weights = false;
+  std::vector<buddy_layer_weights> layers;
+  buddy_dm_weights dm{};
+
+  // scratch (device)
+  float* rope_cos = nullptr;   // [max_pos, hd/2]
+  float* rope_sin = nullptr;
+  int32_t* status = nullptr;   // [0] sticky bits, [1] abort flag, [2..] spare
+  void* xn = nullptr;          // [maxB, d]   act dtype: normalised GEMM input
+  void* act = nullptr;         // [maxB, F]   act dtype: SwiGLU output
+  void* attn_out = nullptr;    // [maxB, qd]  act dtype
+  float* qkv = nullptr;        // [maxB, qkvN]
+  float* q = nullptr;          // [maxB, qd]
+  int attn_chunk = 128, attn_max_chunks = 1;
+  float* attn_m = nullptr;     // [maxB, nq, max_chunks]
+  float* attn_l = nullptr;
+  float* attn_acc = nullptr;   // [maxB, nq, max_chunks, hd]
+  float* dm_u = nullptr;       // [maxB, r]
+  uint8_t* mask = nullptr;     // [maxB, L]
+  int32_t* sel = nullptr;      // [maxB, Lm]
+  float* scores = nullptr;     // [maxB, Lm]
+  int32_t* rows = nullptr;     // [L, maxB]
+  int32_t* count = nullptr;    // [L]
+  // host-buffer entry staging
+  float* h_in_stage = nullptr;
+  float* h_out_stage = nullptr;
+  int32_t* k_stage = nullptr;
+  uint8_t* mask_stage = nullptr;
+
+  // tcgen05 GEMM resources
+  bool use_tc = false;
+  CUtensorMap* tmaps = nullptr;           // device array: per layer 4 weight maps + 3 activation maps
+  std::vector<CUtensorMap> tmaps_host;
+  float* gemm_ws = nullptr;
+  size_t gemm_ws_elems = 0;
+  int32_t* gemm_ctr = nullptr;
+  int gemm_ctr_n = 0;
+
+  // profiler: event pairs around kernel launches (direct-launch mode only)
+  int profiling = 0;
+  struct ProfRec { int cls; int launches; cudaEvent_t a, b; };
+  std::vector<ProfRec> prof;
+  std::vector<cudaEvent_t> ev_pool;
+  size_t ev_used = 0;
+
+  // graph cache
+  int use_graph = 0;
+  struct GraphKey {
+    int B; const void* h_in; const void* k; void* h_out; void* mask; void* rows; void* count;
+    void* scores; cudaStream_t stream; std::vector<const void*> kvp;
+    bool operator<(const GraphKey& o) const;
+  };
+  std::map<GraphKey, cudaGraphExec_t> graphs;
+};
+
+}  // namespace buddy

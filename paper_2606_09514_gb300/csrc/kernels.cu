@@ -1,0 +1,650 @@
+// Non-GEMM kernels of the budget-routed decode step: argument checks, RMSNorm,
+// QKV finalisation (bias, RoPE, cache append, pooled-context update), split-K
+// decode attention, the router (KV-aware pooling + Decision Module + top-k),
+// row compaction with zero K/V for skipped layers, and KV prefill.
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace buddy {
+
+// ---------------------------------------------------------------------------
+// RoPE table: cos/sin of p * theta^(-2j/hd) evaluated in double, stored fp32.
+// ---------------------------------------------------------------------------
+__global__ void rope_table_kernel(float* c, float* s, int max_pos, int hd, double theta) {
+  const int half = hd / 2;
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)max_pos * half) return;
+  const int p = (int)(idx / half), j = (int)(idx % half);
+  const double a = (double)p * pow(theta, -2.0 * (double)j / (double)hd);
+  c[idx] = (float)cos(a);
+  s[idx] = (float)sin(a);
+}
+
+void launch_rope_table(float* c, float* s, int max_pos, int hd, double theta, cudaStream_t st) {
+  const int64_t n = (int64_t)max_pos * (hd / 2);
+  rope_table_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(c, s, max_pos, hd, theta);
+}
+
+// ---------------------------------------------------------------------------
+// Argument checks that need device data.  One CTA decides for the whole call
+// and publishes the abort flag that every later kernel of the call reads.
+// ---------------------------------------------------------------------------
+__global__ void step_check_kernel(int B, const int32_t* k, int Lm, const int32_t* len,
+                                  const int32_t* cap, int extra, int max_pos, int32_t* status) {
+  __shared__ int bad;
+  if (threadIdx.x == 0) bad = 0;
+  __syncthreads();
+  int b = 0;
+  for (int i = threadIdx.x; i < B; i += blockDim.x) {
+    if (k != nullptr) {
+      const int ki = k[i];
+      if (ki < 1 || ki > Lm) b |= BUDDY_DEV_BAD_BUDGET;
+    }
+    const int n = len[i];
+    if (n < 0 || n + extra > cap[i] || n + extra > max_pos) b |= BUDDY_DEV_BAD_POSITION;
+  }
+  if (b) atomicOr(&bad, b);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    status[1] = bad ? 1 : 0;
+    if (bad) atomicOr(status, bad);
+  }
+}
+
+void launch_step_check(const Ctx& c, int B, const int32_t* k, const int32_t* len, const int32_t* cap,
+                       int extra, int32_t* status, cudaStream_t s) {
+  step_check_kernel<<<1, 256, 0, s>>>(B, k, c.Lm, len, cap, extra, c.max_pos, status);
+}
+
+__global__ void kv_check_kernel(int n_seq, const int32_t* ids, int n_new, int batch,
+                                const int32_t* len, const int32_t* cap, int max_pos, int32_t* status) {
+  __shared__ int bad;
+  if (threadIdx.x == 0) bad = 0;
+  __syncthreads();
+  int b = 0;
+  for (int j = threadIdx.x; j < n_seq; j += blockDim.x) {
+    const int s = ids[j];
+    if (s < 0 || s >= batch) {
+      b |= BUDDY_DEV_BAD_SEQ;
+      continue;
+    }
+    const int n = len[s];
+    if (n < 0 || n + n_new > cap[s] || n + n_new > max_pos) b |= BUDDY_DEV_BAD_POSITION;
+  }
+  if (b) atomicOr(&bad, b);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    status[1] = bad ? 1 : 0;
+    if (bad) atomicOr(status, bad);
+  }
+}
+
+void launch_kv_check(const Ctx& c, int n_seq, const int32_t* ids, int n_new, int batch,
+                     const int32_t* len, const int32_t* cap, int32_t* status, cudaStream_t s) {
+  kv_check_kernel<<<1, 256, 0, s>>>(n_seq, ids, n_new, batch, len, cap, c.max_pos, status);
+}
+
+// ---------------------------------------------------------------------------
+// Block-wide sum for 256-thread blocks.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float block_sum_256(float v, float* red) {
+  v = warp_sum(v);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  float t = (l < (int)(blockDim.x >> 5)) ? red[l] : 0.f;
+  t = warp_sum(t);
+  __syncthreads();
+  return t;
+}
+
+// ---------------------------------------------------------------------------
+// RMSNorm with row gather: xn[j] = act(H[rows[j]] * rsqrt(mean(H^2) + eps) * g)
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ H, int d,
+                                                      const int32_t* rows, const int32_t* count, int n,
+                                                      const float* __restrict__ gamma, float eps,
+                                                      T* __restrict__ xn, const int32_t* status) {
+  if (call_aborted(status)) return;
+  const int m = count ? *count : n;
+  const int j = blockIdx.x;
+  if (j >= m) return;
+  const int i = rows ? rows[j] : j;
+  __shared__ float red[32];
+  const float* h = H + (size_t)i * d;
+  float ss = 0.f;
+  for (int e = threadIdx.x * 4; e < d; e += blockDim.x * 4) {
+    const float4 v = *reinterpret_cast<const float4*>(h + e);
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  ss = block_sum_256(ss, red);
+  const float inv = rsqrtf(ss / (float)d + eps);
+  T* o = xn + (size_t)j * d;
+  for (int e = threadIdx.x * 4; e < d; e += blockDim.x * 4) {
+    const float4 v = *reinterpret_cast<const float4*>(h + e);
+    const float4 g = *reinterpret_cast<const float4*>(gamma + e);
+    o[e + 0] = from_f<T>(v.x * inv * g.x);
+    o[e + 1] = from_f<T>(v.y * inv * g.y);
+    o[e + 2] = from_f<T>(v.z * inv * g.z);
+    o[e + 3] = from_f<T>(v.w * inv * g.w);
+  }
+}
+
+void launch_rmsnorm(const Ctx& c, const float* H, RowSel sel, const float* gamma, void* xn,
+                    cudaStream_t s) {
+  if (c.dtype == BUDDY_DTYPE_BF16)
+    rmsnorm_kernel<bf16><<<sel.n, 256, 0, s>>>(H, c.d, sel.rows, sel.count, sel.n, gamma,
+                                               c.cfg.rms_eps, (bf16*)xn, c.status);
+  else
+    rmsnorm_kernel<float><<<sel.n, 256, 0, s>>>(H, c.d, sel.rows, sel.count, sel.n, gamma,
+                                                c.cfg.rms_eps, (float*)xn, c.status);
+}
+
+// ---------------------------------------------------------------------------
+// QKV finalisation for one layer: bias, rotate-half RoPE at position len[i],
+// q kept in fp32, K/V stored (config dtype) at position len[i] of the cache,
+// and for the first layer the pooled-context running sum += stored V.
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(256) qkv_finalize_kernel(
+    const float* __restrict__ qkv, const float* __restrict__ bias, const int32_t* rows,
+    const int32_t* count, int n, int nq, int nkv, int hd, const float* __restrict__ rc,
+    const float* __restrict__ rs, const int32_t* len, const int64_t* seq_off, const int32_t* cap,
+    T* Kc, T* Vc, float* __restrict__ q_out, float* pool, const int32_t* status) {
+  if (call_aborted(status)) return;
+  const int m = count ? *count : n;
+  const int j = blockIdx.x;
+  if (j >= m) return;
+  const int i = rows ? rows[j] : j;
+  const int pos = len[i];
+  const int half = hd / 2;
+  const int N = (nq + 2 * nkv) * hd;
+  const float* x = qkv + (size_t)j * N;
+  const float* cr = rc + (size_t)pos * half;
+  const float* sr = rs + (size_t)pos * half;
+  for (int t = threadIdx.x; t < (nq + nkv) * half; t += blockDim.x) {
+    const int head = t / half, e = t - head * half;
+    const int c0 = head * hd + e;
+    float x1 = x[c0], x2 = x[c0 + half];
+    if (bias) {
+      x1 += bias[c0];
+      x2 += bias[c0 + half];
+    }
+    const float co = cr[e], si = sr[e];
+    const float y1 = x1 * co - x2 * si;
+    const float y2 = x2 * co + x1 * si;
+    if (head < nq) {
+      q_out[(size_t)j * nq * hd + c0] = y1;
+      q_out[(size_t)j * nq * hd + c0 + half] = y2;
+    } else {
+      const int g = head - nq;
+      T* kp = Kc + kv_offset(seq_off, cap, i, nkv, hd, g, pos);
+      kp[e] = from_f<T>(y1);
+      kp[e + half] = from_f<T>(y2);
+    }
+  }
+  const int vbase = (nq + nkv) * hd;
+  for (int t = threadIdx.x; t < nkv * hd; t += blockDim.x) {
+    const int g = t / hd, e = t - g * hd;
+    float v = x[vbase + t];
+    if (bias) v += bias[vbase + t];
+    const T vs = from_f<T>(v);
+    Vc[kv_offset(seq_off, cap, i, nkv, hd, g, pos) + e] = vs;
+    if (pool) pool[(size_t)i * nkv * hd + t] += to_f(vs);
+  }
+}
+
+void launch_qkv_finalize(const Ctx& c, const float* qkv, const float* bias, RowSel sel,
+                         const buddy_kv_state& kv, int layer, float* q_out, float* pool,
+                         cudaStream_t s) {
+  if (c.dtype == BUDDY_DTYPE_BF16)
+    qkv_finalize_kernel<bf16><<<sel.n, 256, 0, s>>>(
+        qkv, bias, sel.rows, sel.count, sel.n, c.nq, c.nkv, c.hd, c.rope_cos, c.rope_sin, kv.len,
+        kv.seq_off, kv.cap, (bf16*)kv.k_cache[layer], (bf16*)kv.v_cache[layer], q_out, pool, c.status);
+  else
+    qkv_finalize_kernel<float><<<sel.n, 256, 0, s>>>(
+        qkv, bias, sel.rows, sel.count, sel.n, c.nq, c.nkv, c.hd, c.rope_cos, c.rope_sin, kv.len,
+        kv.seq_off, kv.cap, (float*)kv.k_cache[layer], (float*)kv.v_cache[layer], q_out, pool,
+        c.status);
+}
+
+// ---------------------------------------------------------------------------
+// Decode attention (Eq. 9) for one layer, split over KV chunks.
+// CTA = (chunk, kv head g, active row j), HD threads.  All G = n_q/n_kv query
+// heads of the group share one pass over the chunk's K and V.  Positions
+// 0..len[i] (the new token included) are attended; zero-filled positions of
+// skipped steps take part with logit 0 (Sec. 6).
+// Partials (running max, sum of exponentials, unnormalised output) per chunk,
+// merged by attn_combine_kernel.
+// ---------------------------------------------------------------------------
+constexpr int kMaxGroup = 8;
+
+template <typename T, int HD>
+__global__ void __launch_bounds__(HD) attn_partial_kernel(
+    const float* __restrict__ q, const int32_t* rows, const int32_t* count, int n, int nq, int nkv,
+    const int32_t* len, const int64_t* seq_off, const int32_t* cap, const T* __restrict__ Kc,
+    const T* __restrict__ Vc, int chunk, int max_chunks, float* __restrict__ part_m,
+    float* __restrict__ part_l, float* __restrict__ part_acc, const int32_t* status) {
+  if (call_aborted(status)) return;
+  const int m = count ? *count : n;
+  const int c = blockIdx.x, g = blockIdx.y, j = blockIdx.z;
+  if (j >= m) return;
+  const int i = rows ? rows[j] : j;
+  const int npos = len[i] + 1;
+  const int p0 = c * chunk;
+  if (p0 >= npos) return;
+  const int p1 = min(npos, p0 + chunk);
+  const int G = nq / nkv;
+  constexpr int NW = HD / 32;
+  constexpr int EPL = HD / 32;  // channels per lane
+  extern __shared__ float sm[];
+  float* qs = sm;                   // [G][HD]
+  float* ss = sm + G * HD;          // [G][chunk]
+  __shared__ float mx_s[kMaxGroup], sum_s[kMaxGroup];
+  const float scale = rsqrtf((float)HD);
+  for (int t = threadIdx.x; t < G * HD; t += HD)
+    qs[t] = q[(size_t)j * nq * HD + (size_t)g * G * HD + t] * scale;
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const T* Kb = Kc + kv_offset(seq_off, cap, i, nkv, HD, g, 0);
+  const T* Vb = Vc + kv_offset(seq_off, cap, i, nkv, HD, g, 0);
+  // logits
+  for (int p = p0 + warp; p < p1; p += NW) {
+    float kv[EPL];
+#pragma unroll
+    for (int u = 0; u < EPL; ++u) kv[u] = to_f(Kb[(size_t)p * HD + lane * EPL + u]);
+    for (int h = 0; h < G; ++h) {
+      float a = 0.f;
+#pragma unroll
+      for (int u = 0; u < EPL; ++u) a += qs[h * HD + lane * EPL + u] * kv[u];
+      a = warp_sum(a);
+      if (lane == 0) ss[h * chunk + (p - p0)] = a;
+    }
+  }
+  __syncthreads();
+  // per-head max and exponentials
+  const int cnt = p1 - p0;
+  for (int h = warp; h < G; h += NW) {
+    float mxv = -INFINITY;
+    for (int t = lane; t < cnt; t += 32) mxv = fmaxf(mxv, ss[h * chunk + t]);
+    mxv = warp_max(mxv);
+    float sv = 0.f;
+    for (int t = lane; t < cnt; t += 32) {
+      const float e = expf(ss[h * chunk + t] - mxv);
+      ss[h * chunk + t] = e;
+      sv += e;
+    }
+    sv = warp_sum(sv);
+    if (lane == 0) {
+      mx_s[h] = mxv;
+      sum_s[h] = sv;
+    }
+  }
+  __syncthreads();
+  // P.V
+  const int e = threadIdx.x;
+  float acc[kMaxGroup];
+#pragma unroll
+  for (int h = 0; h < kMaxGroup; ++h) acc[h] = 0.f;
+  for (int p = p0; p < p1; ++p) {
+    const float v = to_f(Vb[(size_t)p * HD + e]);
+#pragma unroll
+    for (int h = 0; h < kMaxGroup; ++h)
+      if (h < G) acc[h] += ss[h * chunk + (p - p0)] * v;
+  }
+  for (int h = 0; h < G; ++h) {
+    const size_t slot = ((size_t)j * nq + g * G + h) * max_chunks + c;
+    part_acc[slot * HD + e] = acc[h];
+    if (e == 0) {
+      part_m[slot] = mx_s[h];
+      part_l[slot] = sum_s[h];
+    }
+  }
+}
+
+template <typename T, int HD>
+__global__ void __launch_bounds__(HD) attn_combine_kernel(
+    const int32_t* rows, const int32_t* count, int n, int nq, const int32_t* len, int chunk,
+    int max_chunks, const float* __restrict__ part_m, const float* __restrict__ part_l,
+    const float* __restrict__ part_acc, T* __restrict__ out, const int32_t* status) {
+  if (call_aborted(status)) return;
+  const int m = count ? *count : n;
+  const int j = blockIdx.x, h = blockIdx.y;
+  if (j >= m) return;
+  const int i = rows ? rows[j] : j;
+  const int nc = (len[i] + 1 + chunk - 1) / chunk;
+  const size_t base = ((size_t)j * nq + h) * max_chunks;
+  float M = -INFINITY;
+  for (int c = 0; c < nc; ++c) M = fmaxf(M, part_m[base + c]);
+  float Ls = 0.f, a = 0.f;
+  const int e = threadIdx.x;
+  for (int c = 0; c < nc; ++c) {
+    const float w = expf(part_m[base + c] - M);
+    Ls += part_l[base + c] * w;
+    a += part_acc[(base + c) * HD + e] * w;
+  }
+  out[(size_t)j * nq * HD + (size_t)h * HD + e] = from_f<T>(a / Ls);
+}
+
+template <typename T, int HD>
+static void attention_impl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer,
+                           const float* q, void* out, cudaStream_t s) {
+  const int G = c.nq / c.nkv;
+  dim3 grid(c.attn_max_chunks, c.nkv, sel.n);
+  const size_t smem = (size_t)G * (HD + c.attn_chunk) * sizeof(float);
+  attn_partial_kernel<T, HD><<<grid, HD, smem, s>>>(
+      q, sel.rows, sel.count, sel.n, c.nq, c.nkv, kv.len, kv.seq_off, kv.cap,
+      (const T*)kv.k_cache[layer], (const T*)kv.v_cache[layer], c.attn_chunk, c.attn_max_chunks,
+      c.attn_m, c.attn_l, c.attn_acc, c.status);
+  dim3 g2(sel.n, c.nq);
+  attn_combine_kernel<T, HD><<<g2, HD, 0, s>>>(sel.rows, sel.count, sel.n, c.nq, kv.len,
+                                               c.attn_chunk, c.attn_max_chunks, c.attn_m, c.attn_l,
+                                               c.attn_acc, (T*)out, c.status);
+}
+
+void launch_attention(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q,
+                      void* out, cudaStream_t s) {
+  if (c.dtype == BUDDY_DTYPE_BF16) {
+    if (c.hd == 128) attention_impl<bf16, 128>(c, sel, kv, layer, q, out, s);
+    else attention_impl<bf16, 64>(c, sel, kv, layer, q, out, s);
+  } else {
+    if (c.hd == 128) attention_impl<float, 128>(c, sel, kv, layer, q, out, s);
+    else attention_impl<float, 64>(c, sel, kv, layer, q, out, s);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Router, part 1 (Sec. 4.3 + App. C.1 first linear layer):
+//   x_i = [ pool_sum[i] / (len[i] + len_bias), expanded over query heads ; h1[i] ]
+//   u[i][r] = SiLU(b1[r] + W1[r] . x_i)
+// One warp per hidden unit r and up to 8 sequences.
+// ---------------------------------------------------------------------------
+constexpr int kRouteRows = 8;
+
+__global__ void __launch_bounds__(256) route_hidden_kernel(
+    int B, int d, int hd, int group, int nkv, const float* __restrict__ h1,
+    const float* __restrict__ pool, const int32_t* len, int len_bias, const float* __restrict__ w1,
+    const float* __restrict__ b1, int r, float* __restrict__ u, const int32_t* status) {
+  if (call_aborted(status)) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int unit = blockIdx.x * 8 + warp;
+  const int i0 = blockIdx.y * kRouteRows;
+  if (unit >= r) return;
+  const int nr = min(kRouteRows, B - i0);
+  float inv[kRouteRows];
+#pragma unroll
+  for (int t = 0; t < kRouteRows; ++t) inv[t] = (t < nr) ? 1.0f / (float)(len[i0 + t] + len_bias) : 0.f;
+  float acc[kRouteRows];
+#pragma unroll
+  for (int t = 0; t < kRouteRows; ++t) acc[t] = 0.f;
+  const float* wr = w1 + (size_t)unit * 2 * d;
+  const int kvd = nkv * hd;
+  // pooled part: x[k] = pool[(k / hd) / group * hd + k % hd] / n
+  for (int k = lane * 4; k < d; k += 128) {
+    const float4 w = __ldg(reinterpret_cast<const float4*>(wr + k));
+    const int qh = k / hd, e = k - qh * hd;
+    const int pk = (qh / group) * hd + e;
+#pragma unroll
+    for (int t = 0; t < kRouteRows; ++t) {
+      if (t < nr) {
+        const float4 pv = *reinterpret_cast<const float4*>(pool + (size_t)(i0 + t) * kvd + pk);
+        acc[t] += (w.x * pv.x + w.y * pv.y + w.z * pv.z + w.w * pv.w) * inv[t];
+      }
+    }
+  }
+  for (int k = lane * 4; k < d; k += 128) {
+    const float4 w = __ldg(reinterpret_cast<const float4*>(wr + d + k));
+#pragma unroll
+    for (int t = 0; t < kRouteRows; ++t) {
+      if (t < nr) {
+        const float4 hv = *reinterpret_cast<const float4*>(h1 + (size_t)(i0 + t) * d + k);
+        acc[t] += w.x * hv.x + w.y * hv.y + w.z * hv.z + w.w * hv.w;
+      }
+    }
+  }
+#pragma unroll
+  for (int t = 0; t < kRouteRows; ++t) acc[t] = warp_sum(acc[t]);
+  if (lane < nr) {
+    float v = 0.f;
+#pragma unroll
+    for (int t = 0; t < kRouteRows; ++t)
+      if (t == lane) v = acc[t];
+    u[(size_t)(i0 + lane) * r + unit] = silu_f(v + b1[unit]);
+  }
+}
+
+// Router, part 2: s' = W2 u + b2 + omega p~, then the deterministic top-k
+// (Eq. 2): layer l is selected iff fewer than k_i layers rank above it, where
+// l' ranks above l when s'[l'] > s'[l], or s'[l'] == s'[l] and l' < l.
+// One CTA per sequence.
+__global__ void __launch_bounds__(64) route_select_kernel(
+    int Lm, int r, const float* __restrict__ u, const float* __restrict__ w2,
+    const float* __restrict__ b2, const float* __restrict__ prior, float omega, const int32_t* k,
+    uint8_t* mask, int32_t* sel, float* scores, const int32_t* status) {
+  if (call_aborted(status)) return;
+  const int i = blockIdx.x;
+  extern __shared__ float s[];           // [Lm]
+  __shared__ int flag[kMaxLayers];
+  const float* ui = u + (size_t)i * r;
+  for (int l = threadIdx.x; l < Lm; l += blockDim.x) {
+    float a = 0.f;
+    const float* w = w2 + (size_t)l * r;
+    for (int t = 0; t < r; ++t) a += w[t] * ui[t];
+    a += b2[l];
+    if (prior) a += omega * prior[l];
+    s[l] = a;
+  }
+  __syncthreads();
+  const int ki = k[i];
+  for (int l = threadIdx.x; l < Lm; l += blockDim.x) {
+    int rank = 0;
+    const float v = s[l];
+    for (int t = 0; t < Lm; ++t) rank += (s[t] > v) || (s[t] == v && t < l);
+    flag[l] = rank < ki;
+  }
+  __syncthreads();
+  const int L = Lm + 2;
+  for (int l = threadIdx.x; l < Lm; l += blockDim.x) {
+    if (scores) scores[(size_t)i * Lm + l] = s[l];
+    if (mask) mask[(size_t)i * L + l + 1] = (uint8_t)flag[l];
+    if (sel) {
+      int before = 0;
+      for (int t = 0; t < l; ++t) before += flag[t];
+      if (flag[l]) sel[(size_t)i * Lm + before] = l + 1;
+      if (l >= ki) sel[(size_t)i * Lm + l] = -1;
+    }
+  }
+  if (threadIdx.x == 0 && mask) {
+    mask[(size_t)i * L] = 1;
+    mask[(size_t)i * L + L - 1] = 1;
+  }
+}
+
+void launch_route(const Ctx& c, int B, const float* h1, const float* pool, const int32_t* len,
+                  int len_bias, const int32_t* k, uint8_t* mask, int32_t* sel, float* scores,
+                  cudaStream_t s) {
+  dim3 g1((c.r + 7) / 8, (B + kRouteRows - 1) / kRouteRows);
+  route_hidden_kernel<<<g1, 256, 0, s>>>(B, c.d, c.hd, c.nq / c.nkv, c.nkv, h1, pool, len, len_bias,
+                                         c.dm.w1, c.dm.b1, c.r, c.dm_u, c.status);
+  route_select_kernel<<<B, 64, c.Lm * sizeof(float), s>>>(c.Lm, c.r, c.dm_u, c.dm.w2, c.dm.b2,
+                                                          c.dm.prior, c.dm.omega, k, mask, sel,
+                                                          scores, c.status);
+}
+
+// ---------------------------------------------------------------------------
+// Grouping by mask (App. C.1): per layer, the ascending list of sequences that
+// execute it and their number (exclusive prefix sum over the mask column).
+// Sequences that skip a middle layer get zero K and V at their new position
+// in that layer (Sec. 6).  One CTA per layer.
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(1024) compact_kernel(int B, int L, int nkv, int hd,
+                                                       const uint8_t* __restrict__ mask,
+                                                       LayerPtrs ptrs, const int32_t* len,
+                                                       const int64_t* seq_off, const int32_t* cap,
+                                                       int32_t* rows, int32_t* count,
+                                                       const int32_t* status) {
+  if (call_aborted(status)) return;
+  const int l = blockIdx.x;
+  int32_t* rl = rows + (size_t)l * B;
+  __shared__ int wsum[32];
+  __shared__ int carry;
+  if (threadIdx.x == 0) carry = 0;
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  for (int base = 0; base < B; base += blockDim.x) {
+    const int i = base + threadIdx.x;
+    const int f = (i < B) ? mask[(size_t)i * L + l] : 0;
+    const unsigned bal = __ballot_sync(0xffffffffu, f);
+    const int before_in_warp = __popc(bal & ((1u << lane) - 1u));
+    if (lane == 0) wsum[warp] = __popc(bal);
+    __syncthreads();
+    int before_warps = 0;
+    for (int w = 0; w < warp; ++w) before_warps += wsum[w];
+    if (f) rl[carry + before_warps + before_in_warp] = i;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int tot = 0;
+      for (int w = 0; w < nw; ++w) tot += wsum[w];
+      carry += tot;
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) count[l] = carry;
+  // zero K/V at the new position for sequences that skip this layer
+  if (l == 0 || l == L - 1) return;
+  T* Kc = (T*)ptrs.k[l];
+  T* Vc = (T*)ptrs.v[l];
+  const int kvd = nkv * hd;
+  for (int i = 0; i < B; ++i) {
+    if (mask[(size_t)i * L + l]) continue;
+    const int pos = len[i];
+    for (int t = threadIdx.x; t < kvd; t += blockDim.x) {
+      const int g = t / hd, e = t - g * hd;
+      const int64_t off = kv_offset(seq_off, cap, i, nkv, hd, g, pos) + e;
+      Kc[off] = from_f<T>(0.f);
+      Vc[off] = from_f<T>(0.f);
+    }
+  }
+}
+
+void launch_compact(const Ctx& c, int B, const uint8_t* mask, const buddy_kv_state& kv,
+                    int32_t* rows, int32_t* count, cudaStream_t s) {
+  LayerPtrs p;
+  for (int l = 0; l < c.L; ++l) {
+    p.k[l] = kv.k_cache[l];
+    p.v[l] = kv.v_cache[l];
+  }
+  if (c.dtype == BUDDY_DTYPE_BF16)
+    compact_kernel<bf16><<<c.L, 1024, 0, s>>>(B, c.L, c.nkv, c.hd, mask, p, kv.len, kv.seq_off,
+                                              kv.cap, rows, count, c.status);
+  else
+    compact_kernel<float><<<c.L, 1024, 0, s>>>(B, c.L, c.nkv, c.hd, mask, p, kv.len, kv.seq_off,
+                                               kv.cap, rows, count, c.status);
+}
+
+// ---------------------------------------------------------------------------
+// Position advance: len[i] += by  (for i < B, or for the listed sequences).
+// ---------------------------------------------------------------------------
+__global__ void advance_kernel(int B, int32_t* len, int by, const int32_t* ids,
+                               const int32_t* status) {
+  if (call_aborted(status)) return;
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= B) return;
+  const int i = ids ? ids[t] : t;
+  len[i] += by;
+}
+
+void launch_advance(const Ctx& c, int B, int32_t* len, int by, const int32_t* ids, cudaStream_t s) {
+  advance_kernel<<<(B + 255) / 256, 256, 0, s>>>(B, len, by, ids, c.status);
+}
+
+// ---------------------------------------------------------------------------
+// Prefill / bulk append of positions to one layer (Eq. 9), and the full
+// recomputation of the pooled first-layer context for the appended sequences.
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(256) kv_append_kernel(int n_new, int nkv, int hd,
+                                                        const int32_t* ids, const int32_t* len,
+                                                        const int64_t* seq_off, const int32_t* cap,
+                                                        const T* __restrict__ kn,
+                                                        const T* __restrict__ vn, T* Kc, T* Vc,
+                                                        const int32_t* status) {
+  if (call_aborted(status)) return;
+  const int t = blockIdx.x, jj = blockIdx.y;
+  const int s = ids[jj];
+  const int pos = len[s] + t;
+  const int kvd = nkv * hd;
+  const size_t src = ((size_t)jj * n_new + t) * kvd;
+  for (int x = threadIdx.x; x < kvd; x += blockDim.x) {
+    const int g = x / hd, e = x - g * hd;
+    const int64_t off = kv_offset(seq_off, cap, s, nkv, hd, g, pos) + e;
+    Kc[off] = kn[src + x];
+    Vc[off] = vn[src + x];
+  }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) pool_refresh_kernel(int n_new, int nkv, int hd,
+                                                           const int32_t* ids, const int32_t* len,
+                                                           const int64_t* seq_off,
+                                                           const int32_t* cap, const T* V0,
+                                                           float* pool, const int32_t* status) {
+  if (call_aborted(status)) return;
+  const int s = ids[blockIdx.y];
+  const int kvd = nkv * hd;
+  const int x = blockIdx.x * blockDim.x + threadIdx.x;
+  if (x >= kvd) return;
+  const int g = x / hd, e = x - g * hd;
+  const int n = len[s] + n_new;
+  const T* base = V0 + kv_offset(seq_off, cap, s, nkv, hd, g, 0) + e;
+  float acc = 0.f;
+  for (int p = 0; p < n; ++p) acc += to_f(base[(size_t)p * hd]);
+  pool[(size_t)s * kvd + x] = acc;
+}
+
+void launch_kv_append(const Ctx& c, const buddy_kv_state& kv, int layer, int n_seq,
+                      const int32_t* ids, int n_new, const void* kn, const void* vn, cudaStream_t s) {
+  dim3 g(n_new, n_seq);
+  if (c.dtype == BUDDY_DTYPE_BF16)
+    kv_append_kernel<bf16><<<g, 256, 0, s>>>(n_new, c.nkv, c.hd, ids, kv.len, kv.seq_off, kv.cap,
+                                             (const bf16*)kn, (const bf16*)vn,
+                                             (bf16*)kv.k_cache[layer], (bf16*)kv.v_cache[layer],
+                                             c.status);
+  else
+    kv_append_kernel<float><<<g, 256, 0, s>>>(n_new, c.nkv, c.hd, ids, kv.len, kv.seq_off, kv.cap,
+                                              (const float*)kn, (const float*)vn,
+                                              (float*)kv.k_cache[layer], (float*)kv.v_cache[layer],
+                                              c.status);
+}
+
+void launch_pool_refresh(const Ctx& c, const buddy_kv_state& kv, int n_seq, const int32_t* ids,
+                         int n_new, cudaStream_t s) {
+  dim3 g((c.kvd + 255) / 256, n_seq);
+  if (c.dtype == BUDDY_DTYPE_BF16)
+    pool_refresh_kernel<bf16><<<g, 256, 0, s>>>(n_new, c.nkv, c.hd, ids, kv.len, kv.seq_off, kv.cap,
+                                                (const bf16*)kv.v_cache[0], kv.pool_sum, c.status);
+  else
+    pool_refresh_kernel<float><<<g, 256, 0, s>>>(n_new, c.nkv, c.hd, ids, kv.len, kv.seq_off,
+                                                 kv.cap, (const float*)kv.v_cache[0], kv.pool_sum,
+                                                 c.status);
+}
+
+// ---------------------------------------------------------------------------
+// Graph conditional: execute a layer's body iff some sequence selected it.
+// ---------------------------------------------------------------------------
+__global__ void set_conditional_kernel(cudaGraphConditionalHandle h, const int32_t* count,
+                                       const int32_t* status) {
+  const bool run = !call_aborted(status) && *count > 0;
+  cudaGraphSetConditional(h, run ? 1u : 0u);
+}
+
+void launch_set_conditional(cudaGraphConditionalHandle h, const int32_t* count,
+                            const int32_t* status, cudaStream_t s) {
+  set_conditional_kernel<<<1, 1, 0, s>>>(h, count, status);
+}
+
+}  // namespace buddy

@@ -1,0 +1,59 @@
+"""Parity rules between the GPU path and the oracle.
+
+* Routes: the GPU's selected set must equal the oracle's, except when the
+  oracle's k-th and (k+1)-th scores differ by less than ROUTE_MARGIN: then the
+  oracle adopts the GPU's set, provided every layer on which the two sets
+  differ has an oracle score within ROUTE_MARGIN of the k-th score.
+* Hidden states: per sequence, max_j |g_j - o_j| / max_j |o_j| below
+  HIDDEN_TOL[dtype].
+* Compaction indices (rows/count): bit-exact against the oracle's grouping of
+  the (adopted) selections.
+"""
+from __future__ import annotations
+
+from typing import List, Sequence, Tuple
+
+import numpy as np
+
+ROUTE_MARGIN = 1e-3
+HIDDEN_TOL = {"f32": 1e-4, "bf16": 2e-2}
+
+
+def adopt_routes(o_scores: np.ndarray, o_sel: Sequence[Sequence[int]], g_sel: Sequence[Sequence[int]],
+                 k: Sequence[int]) -> Tuple[List[List[int]], List[str], int]:
+    """Returns (sets the oracle continues with, failures, number adopted)."""
+    out, fails, adopted = [], [], 0
+    for i, (os_, gs) in enumerate(zip(o_sel, g_sel)):
+        os_, gs = sorted(int(x) for x in os_), sorted(int(x) for x in gs)
+        if os_ == gs:
+            out.append(os_)
+            continue
+        s = np.asarray(o_scores[i], dtype=np.float64)
+        ki = int(k[i])
+        srt = np.sort(s)[::-1]
+        if len(gs) != ki or ki >= len(s):
+            fails.append(f"seq {i}: gpu {gs} vs oracle {os_} (k={ki})")
+            out.append(os_)
+            continue
+        kth = srt[ki - 1]
+        gap = srt[ki - 1] - srt[ki]
+        diff = set(os_) ^ set(gs)
+        near = all(abs(s[l - 1] - kth) < ROUTE_MARGIN for l in diff)
+        if gap < ROUTE_MARGIN and near:
+            out.append(gs)
+            adopted += 1
+        else:
+            fails.append(f"seq {i}: gpu {gs} vs oracle {os_}, gap {gap:.3g}")
+            out.append(os_)
+    return out, fails, adopted
+
+
+def max_rel_err(g: np.ndarray, o: np.ndarray) -> float:
+    g = np.asarray(g, dtype=np.float64)
+    o = np.asarray(o, dtype=np.float64)
+    return float(np.max(np.abs(g - o)) / max(np.max(np.abs(o)), 1e-30))
+
+
+def sel_from_mask(mask: np.ndarray) -> List[List[int]]:
+    L = mask.shape[1]
+    return [[l for l in range(1, L - 1) if mask[i, l]] for i in range(mask.shape[0])]

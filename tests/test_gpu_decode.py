@@ -1,0 +1,257 @@
+"""GPU parity: libbuddy's decode step (through the C ABI) against the oracle.
+
+Small workloads that span several GEMM tiles with ragged tails, contexts 0..1000
+(including n_i = 0 and chunk boundaries), budgets 1..L_mid, GQA groups 1..4,
+qkv bias on/off, fp32 and bf16.  Multi-step runs are free-running on both
+sides; the near-tie rule is the only place the oracle takes a GPU decision.
+"""
+import numpy as np
+import pytest
+import torch
+
+import parity as P
+from oracle import adapter as A
+from oracle import buddy_oracle as O
+from workloads import configs as C
+from workloads import device as D
+from workloads import synth
+
+pytestmark = pytest.mark.gpu
+
+
+def _oracle_for(dw, gen_device="cuda"):
+    w = dw.w
+    s = w.shape
+    model = A.build_model(s, w.seed, layer_source=lambda l: synth.layer_weights(s, w.seed, l, gen_device),
+                          dm_source=lambda: synth.dm_weights(s, w.seed, gen_device),
+                          prior=dw.prior, omega=0.1 if dw.prior is not None else 0.0,
+                          cache_layers=s.n_layers)
+    st = A.build_state(s, w.seed, w.contexts(), gen_device=gen_device)
+    return model, st
+
+
+def run_parity(w, steps=None, use_graph=False, prior=False, check_kv=True):
+    dw = D.build(w, use_graph=use_graph, prior=prior)
+    model, st = _oracle_for(dw)
+    s = w.shape
+    B, L, Lm = w.batch, s.n_layers, s.l_mid
+    dev = "cuda"
+    h_out = torch.empty(B, s.d_model, device=dev)
+    mask = torch.empty(B, L, dtype=torch.uint8, device=dev)
+    rows = torch.empty(L, B, dtype=torch.int32, device=dev)
+    count = torch.empty(L, dtype=torch.int32, device=dev)
+    scores = torch.empty(B, Lm, device=dev)
+    k = w.budgets()
+    tol = P.HIDDEN_TOL[s.dtype]
+    worst = 0.0
+    adopted_total = 0
+    for t in range(steps or w.steps):
+        n_before = list(st.n)
+        h_in = synth.workload_h_in(w, t, dev)
+        dw.ctx.buddy_decode_step(dw.kv, h_in, dw.k, h_out, mask, rows, count, scores)
+        torch.cuda.synchronize()
+        assert dw.ctx.buddy_device_status() == 0
+        g_mask = mask.cpu().numpy()
+        g_sel = P.sel_from_mask(g_mask)
+        info = {}
+
+        def override(route):
+            sel, fails, n = P.adopt_routes(route.scores, route.sel, g_sel, k)
+            info["fails"], info["n"] = fails, n
+            return sel
+
+        res = O.decode_step(model, st, A.to_f64(h_in), k, override_sel=override)
+        assert not info["fails"], info["fails"]
+        adopted_total += info["n"]
+        # scores agree well inside the near-tie margin
+        np.testing.assert_allclose(scores.cpu().numpy(), res.scores, rtol=0, atol=P.ROUTE_MARGIN / 4)
+        # exactly k middle layers + first + last
+        np.testing.assert_array_equal(g_mask.sum(1), k + 2)
+        # compaction: bit-exact
+        g_count = count.cpu().numpy()
+        g_rows = rows.cpu().numpy()
+        for l in range(L):
+            assert g_count[l] == len(res.rows[l]), (t, l)
+            assert g_rows[l, : g_count[l]].tolist() == res.rows[l], (t, l)
+        # hidden states
+        g_h = h_out.cpu().numpy()
+        for i in range(B):
+            e = P.max_rel_err(g_h[i], res.h_out[i])
+            worst = max(worst, e)
+            assert e < tol, (t, i, e)
+        # KV written this step: real entries match, skipped layers hold zeros
+        if check_kv:
+            for l in range(L):
+                for i in range(B):
+                    pos = n_before[i]
+                    gk = dw.kv.view("k", l, i)[:, pos, :].float().cpu().numpy()
+                    gv = dw.kv.view("v", l, i)[:, pos, :].float().cpu().numpy()
+                    ok, ov = res.kv_new[(l, i)]
+                    if g_mask[i, l]:
+                        assert P.max_rel_err(gk, ok) < 2 * 2.0 ** -8 and P.max_rel_err(gv, ov) < 2 * 2.0 ** -8
+                    else:
+                        assert not gk.any() and not gv.any()
+    # positions advanced by one per step
+    np.testing.assert_array_equal(dw.kv.len.cpu().numpy(), np.asarray(st.n))
+    return worst, adopted_total
+
+
+@pytest.mark.parametrize("w", [C.T_F32, C.C1_TINY], ids=lambda w: w.name)
+def test_decode_parity_f32(w):
+    worst, _ = run_parity(w, steps=2)
+    assert worst < 1e-4
+
+
+@pytest.mark.parametrize("w", [C.T_GQA, C.T_QWEN], ids=lambda w: w.name)
+def test_decode_parity_bf16(w):
+    worst, _ = run_parity(w)
+    assert worst < 2e-2
+
+
+def test_decode_parity_prior_and_graph():
+    run_parity(C.T_GQA, steps=2, use_graph=True, prior=True)
+
+
+def test_full_budget_every_layer_executes():
+    w = C.scaled(C.T_QWEN, k=[C.T_QWEN.shape.l_mid] * C.T_QWEN.batch, name="t-qwen-dense")
+    run_parity(w, steps=1)
+
+
+def test_budget_one_and_batch_one():
+    w = C.scaled(C.T_GQA, ctx=[77], k=[1], name="t-gqa-b1")
+    run_parity(w, steps=3)
+
+
+def test_graph_replay_equals_direct_launches():
+    w = C.T_GQA
+    outs = []
+    for g in (False, True):
+        dw = D.build(w, use_graph=g)
+        h_out = torch.empty(w.batch, w.shape.d_model, device="cuda")
+        mask = torch.empty(w.batch, w.shape.n_layers, dtype=torch.uint8, device="cuda")
+        res = []
+        for t in range(3):
+            dw.ctx.buddy_decode_step(dw.kv, synth.workload_h_in(w, t, "cuda"), dw.k, h_out, mask)
+            res.append((h_out.clone(), mask.clone()))
+        torch.cuda.synchronize()
+        outs.append(res)
+    for (a, ma), (b, mb) in zip(*outs):
+        assert torch.equal(ma, mb)
+        assert torch.equal(a, b)
+
+
+def test_route_entry_point_matches_oracle_router():
+    """buddy_route alone: pool over the cached first-layer V (including the
+    newest token, already appended), Decision Module, top-k."""
+    w = C.T_QWEN
+    dw = D.build(w, prior=True)
+    s = w.shape
+    B, Lm = w.batch, s.l_mid
+    h1 = synth.h_in(s, 99, 0, range(B), "cuda") * 3.0
+    sel = torch.empty(B, Lm, dtype=torch.int32, device="cuda")
+    mask = torch.empty(B, s.n_layers, dtype=torch.uint8, device="cuda")
+    sc = torch.empty(B, Lm, device="cuda")
+    # the router needs len >= 1: sequences with n_i = 0 get one appended position
+    ctxs = w.contexts()
+    empty = [i for i in range(B) if ctxs[i] == 0]
+    for i in empty:
+        ids = torch.tensor([i], dtype=torch.int32, device="cuda")
+        K = synth.kv_block(s, w.seed, "k", 0, i, 0, 1, "cuda").unsqueeze(0)
+        V = synth.kv_block(s, w.seed, "v", 0, i, 0, 1, "cuda").unsqueeze(0)
+        dw.ctx.buddy_kv_append(dw.kv, 0, ids, K, V, advance=True)
+    dw.ctx.buddy_route(dw.kv, h1, dw.k, sel, mask, sc)
+    torch.cuda.synchronize()
+    assert dw.ctx.buddy_device_status() == 0
+    model, _ = _oracle_for(dw)
+    sh = model.shape
+    lens = dw.kv.len.cpu().numpy()
+    o_sel, o_sc = [], []
+    for i in range(B):
+        V0 = A.to_f64(synth.kv_block(s, w.seed, "v", 0, i, 0, int(lens[i]), "cuda"))
+        x = np.concatenate([O.expand_kv_heads(O.pool_context(V0), sh), A.to_f64(h1[i])])
+        sc_i = O.decision_scores(model.dm, x)
+        o_sc.append(sc_i)
+        o_sel.append(O.top_k_layers(sc_i, int(w.budgets()[i])))
+    o_sc = np.array(o_sc)
+    np.testing.assert_allclose(sc.cpu().numpy(), o_sc, rtol=0, atol=1e-5)
+    g_sel = [[int(v) for v in row if v >= 0] for row in sel.cpu().numpy()]
+    _, fails, _ = P.adopt_routes(o_sc, o_sel, g_sel, w.budgets())
+    assert not fails
+    np.testing.assert_array_equal(mask.cpu().numpy().sum(1), w.budgets() + 2)
+
+
+def test_kv_append_pool_is_full_sum():
+    w = C.T_GQA
+    dw = D.build(w)
+    s = w.shape
+    pool = dw.kv.pool_sum.cpu().numpy().astype(np.float64)
+    for i in range(w.batch):
+        n = int(w.contexts()[i])
+        V0 = A.to_f64(synth.kv_block(s, w.seed, "v", 0, i, 0, n, "cuda")) if n else np.zeros((0, s.n_kv_heads, s.head_dim))
+        ref = V0.sum(0).reshape(-1)
+        np.testing.assert_allclose(pool[i], ref, rtol=1e-5, atol=1e-4)
+    np.testing.assert_array_equal(dw.kv.len.cpu().numpy(), w.contexts())
+
+
+def test_device_checks_write_nothing():
+    w = C.T_GQA
+    dw = D.build(w)
+    s = w.shape
+    B = w.batch
+    h_in = synth.workload_h_in(w, 0, "cuda")
+    h_out = torch.full((B, s.d_model), 7.0, device="cuda")
+    k0 = [t.clone() for t in dw.kv.k]
+    len0 = dw.kv.len.clone()
+    pool0 = dw.kv.pool_sum.clone()
+    bad = dw.k.clone()
+    bad[3] = s.l_mid + 1
+    dw.ctx.buddy_decode_step(dw.kv, h_in, bad, h_out)
+    flags = dw.ctx.buddy_device_status()
+    assert flags & 1
+    assert torch.all(h_out == 7.0)
+    assert torch.equal(dw.kv.len, len0) and torch.equal(dw.kv.pool_sum, pool0)
+    assert all(torch.equal(a, b) for a, b in zip(k0, dw.kv.k))
+    # a position beyond capacity
+    dw.kv.len[5] = int(dw.caps[5])
+    dw.ctx.buddy_decode_step(dw.kv, h_in, dw.k, h_out)
+    assert dw.ctx.buddy_device_status() & 2
+    assert torch.all(h_out == 7.0)
+    # the context stays usable: a valid call succeeds afterwards
+    dw.kv.len.copy_(len0)
+    dw.ctx.buddy_decode_step(dw.kv, h_in, dw.k, h_out)
+    assert dw.ctx.buddy_device_status() == 0
+    assert not torch.all(h_out == 7.0)
+
+
+def test_host_buffer_entry_matches_device_entry():
+    w = C.T_GQA
+    outs = []
+    for host in (False, True):
+        dw = D.build(w)
+        h_in = synth.workload_h_in(w, 0, "cuda")
+        if host:
+            hh = h_in.cpu().pin_memory()
+            kh = dw.k.cpu().pin_memory()
+            oh = torch.empty(w.batch, w.shape.d_model).pin_memory()
+            mh = torch.empty(w.batch, w.shape.n_layers, dtype=torch.uint8).pin_memory()
+            dw.ctx.buddy_decode_step_host(dw.kv, hh, kh, oh, mh)
+            outs.append((oh.clone(), mh.clone()))
+        else:
+            o = torch.empty(w.batch, w.shape.d_model, device="cuda")
+            m = torch.empty(w.batch, w.shape.n_layers, dtype=torch.uint8, device="cuda")
+            dw.ctx.buddy_decode_step(dw.kv, h_in, dw.k, o, m)
+            outs.append((o.cpu(), m.cpu()))
+    assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+
+
+def test_generator_identical_on_cpu_and_gpu():
+    s = C.LLAMA3_8B
+    for kind, ids, n, start in [("w_q", (3,), 100003, 77), ("k_cache", (0, 5), 65536, 1 << 20),
+                                ("h_in", (2, 1), 4096, 0)]:
+        key = synth.stream_key(0, kind, *ids)
+        a = synth.normal((n,), key, 0.02, torch.bfloat16, "cpu", start=start)
+        b = synth.normal((n,), key, 0.02, torch.bfloat16, "cuda", start=start).cpu()
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+        a = synth.normal((n,), key, 1.0, torch.float32, "cpu", start=start)
+        b = synth.normal((n,), key, 1.0, torch.float32, "cuda", start=start).cpu()
+        assert torch.equal(a.view(torch.int32), b.view(torch.int32))
