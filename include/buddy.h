@@ -161,6 +161,34 @@ BUDDY_API int buddy_route(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t batc
                 const int32_t* k, int32_t* sel_out, uint8_t* mask_out, float* scores_out,
                 void* stream);
 
+/* Allocation-free router, for callers that cannot allocate device memory and
+ * therefore cannot create a buddy_ctx: for example a process whose device
+ * memory is all owned by its own pool allocator, or code that runs where
+ * cudaMalloc (which may synchronise the device) is not allowed.  The paper
+ * has no counterpart; this is a deployment variant of buddy_route.
+ *
+ * Computes exactly what buddy_route computes, from explicit arguments instead
+ * of a context: shape (n_layers, d_model, n_q_heads, n_kv_heads, head_dim,
+ * dm_hidden, same rules as buddy_config), Decision Module `dm`, and device
+ * arrays pool_sum [batch, n_kv*hd], len [batch] (>= 1, the cache already holds
+ * the newest token), h1 [batch, d] fp32, k [batch].  Outputs as buddy_route;
+ * flags_out (device int32, may be NULL) receives the BUDDY_DEV_* bits of this
+ * call (0 when valid; on a nonzero value nothing else was written).
+ *
+ * Scratch: one static device array of the library (256 KiB of hidden units
+ * plus a small header), held by every GPU that loads the library until the
+ * process exits.  batch * dm_hidden must not exceed 65536, else
+ * BUDDY_ERR_RANGE.  The first call on each device looks up the array's
+ * device address (cudaGetSymbolAddress); make that first call outside any
+ * stream capture.  All calls share the array: calls whose kernels overlap on
+ * the GPU (different streams without ordering) race.  Allocates nothing. */
+BUDDY_API int buddy_route_noalloc(int32_t n_layers, int32_t d_model, int32_t n_q_heads,
+                                  int32_t n_kv_heads, int32_t head_dim, int32_t dm_hidden,
+                                  const buddy_dm_weights* dm, int32_t batch, const float* pool_sum,
+                                  const int32_t* len, const float* h1, const int32_t* k,
+                                  int32_t* sel_out, uint8_t* mask_out, float* scores_out,
+                                  int32_t* flags_out, void* stream);
+
 /* One budget-routed decode step for sequences 0..batch-1 of `kv`.
  * h_in: device [batch, d] fp32 (input of the first block); k: device [batch]
  * int32 budgets in [1, L-2]; h_out: device [batch, d] fp32, the hidden state

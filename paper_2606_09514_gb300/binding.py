@@ -19,7 +19,8 @@ BUDDY_DEV_BAD_BUDGET, BUDDY_DEV_BAD_POSITION, BUDDY_DEV_BAD_SEQ, BUDDY_DEV_TIMEO
 EXPORTED = ["buddy_create", "buddy_destroy", "buddy_set_weights", "buddy_kv_append", "buddy_route",
             "buddy_decode_step", "buddy_decode_step_host", "buddy_set_options",
             "buddy_device_status", "buddy_budget_to_k", "buddy_error_string", "buddy_version",
-            "buddy_set_profiling", "buddy_profile_read", "buddy_profile_class_name"]
+            "buddy_set_profiling", "buddy_profile_read", "buddy_profile_class_name",
+            "buddy_route_noalloc"]
 PROF_CLASSES = ["check", "rmsnorm", "gemm_qkv", "qkv_finalize", "attention", "gemm_o", "gemm_gate_up",
                 "gemm_down", "route", "compact", "other"]
 
@@ -89,6 +90,9 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.buddy_profile_read.argtypes = [c_p, c_i32, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(c_i32)]
     lib.buddy_profile_class_name.argtypes = [c_i32]
     lib.buddy_profile_class_name.restype = ctypes.c_char_p
+    lib.buddy_route_noalloc.argtypes = [c_i32, c_i32, c_i32, c_i32, c_i32, c_i32, ctypes.POINTER(buddy_dm_weights),
+                                        c_i32, c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p]
+    lib.buddy_route_noalloc.restype = ctypes.c_int
     for name in ("buddy_create", "buddy_set_weights", "buddy_kv_append", "buddy_route", "buddy_decode_step",
                  "buddy_decode_step_host", "buddy_set_options", "buddy_device_status", "buddy_set_profiling",
                  "buddy_profile_read"):
@@ -114,6 +118,21 @@ def _check(rc: int, what: str):
 
 def buddy_budget_to_k(b: float, n_layers: int) -> int:
     return int(load_library().buddy_budget_to_k(float(b), int(n_layers)))
+
+
+def buddy_route_noalloc(shape, dm: Dict[str, torch.Tensor], pool_sum: torch.Tensor, length: torch.Tensor,
+                        h1: torch.Tensor, k: torch.Tensor, sel_out=None, mask_out=None, scores_out=None,
+                        flags_out=None, prior: Optional[torch.Tensor] = None, omega: float = 0.0,
+                        stream=None):
+    """Context-free router (no device allocation); see include/buddy.h."""
+    lib = load_library()
+    dmw = buddy_dm_weights(dm["w1"].data_ptr(), dm["b1"].data_ptr(), dm["w2"].data_ptr(), dm["b2"].data_ptr(),
+                           None if prior is None else prior.data_ptr(), float(omega))
+    _check(lib.buddy_route_noalloc(shape.n_layers, shape.d_model, shape.n_q_heads, shape.n_kv_heads,
+                                   shape.head_dim, shape.dm_hidden, ctypes.byref(dmw), h1.shape[0],
+                                   _ptr(pool_sum), _ptr(length), _ptr(h1), _ptr(k), _ptr(sel_out),
+                                   _ptr(mask_out), _ptr(scores_out), _ptr(flags_out), _stream(stream)),
+           "buddy_route_noalloc")
 
 
 class KVCache:
