@@ -174,6 +174,28 @@ def oracle_sample(w, n_layers_sample=None, steps=1, device="cuda"):
             "cores": os.cpu_count()}
 
 
+def class_bytes(s, masks, ctxs, B):
+    """Algorithmic bytes per kernel class over the profiled steps: weights of
+    every launched layer, activations in and out, KV read by attention."""
+    esz = s.elem_bytes
+    d, F, qd, kvd, N = s.d_model, s.ffn_dim, s.q_dim, s.kv_dim, s.qkv_dim
+    out = {"gemm_gate_up": 0, "gemm_down": 0, "gemm_qkv": 0, "gemm_o": 0, "attention": 0, "rmsnorm": 0}
+    for m_, n_ in zip(masks, ctxs):
+        rows = m_.sum(axis=0)
+        for l in range(s.n_layers):
+            m = int(rows[l])
+            if m == 0:
+                continue
+            out["gemm_gate_up"] += 2 * F * d * esz + m * (d + F) * esz
+            out["gemm_down"] += F * d * esz + m * (F * esz + 8 * d)
+            out["gemm_qkv"] += N * d * esz + m * (d * esz + 4 * N)
+            out["gemm_o"] += qd * d * esz + m * (qd * esz + 8 * d)
+            sel = np.nonzero(m_[:, l])[0]
+            out["attention"] += int(2 * kvd * esz * (n_[:B][sel] + 1).sum()) + m * qd * (4 + esz)
+            out["rmsnorm"] += 2 * m * d * (4 + esz)
+    return out
+
+
 # ---------------------------------------------------------------------------
 # Our arm
 # ---------------------------------------------------------------------------
@@ -273,22 +295,12 @@ def run_ours(args, ws, rank, local):
         for key in c_sum:
             c_sum[key] += c[key]
     prof_ms_total = sum(v[0] for v in prof.values())
-    # dominant kernel class and its algorithmic bytes per launch
+    # dominant kernel class and its algorithmic bytes (summed over the profiled steps)
     dom = max(prof, key=lambda k: prof[k][0])
-    esz = s.elem_bytes
-    rows_per_layer = [m_.sum(axis=0) for m_ in prof_masks]
-    exec_layers = [(r > 0) for r in rows_per_layer]
-    n_launch_layers = int(sum(e.sum() for e in exec_layers))
-    m_sum = int(sum(r.sum() for r in rows_per_layer))
-    per_class_bytes = {
-        "gemm_gate_up": 2 * s.ffn_dim * s.d_model * esz * n_launch_layers + m_sum * (s.d_model + s.ffn_dim) * esz,
-        "gemm_down": s.ffn_dim * s.d_model * esz * n_launch_layers + m_sum * (s.ffn_dim * esz + 8 * s.d_model),
-        "gemm_qkv": s.qkv_dim * s.d_model * esz * n_launch_layers + m_sum * (s.d_model * esz + 4 * s.qkv_dim),
-        "gemm_o": s.q_dim * s.d_model * esz * n_launch_layers + m_sum * (s.q_dim * esz + 8 * s.d_model),
-    }
+    per_class_bytes = class_bytes(s, prof_masks, prof_ctx, B)
     roof = None
     if dom in per_class_bytes and prof[dom][1] > 0:
-        launches = prof[dom][1]
+        launches = prof[dom][1] if dom != "attention" else prof[dom][1] // 2
         bytes_per_launch = per_class_bytes[dom] / launches
         avg_s = prof[dom][0] / 1e3 / launches
         ach = bytes_per_launch / avg_s / 1e9
@@ -317,6 +329,8 @@ def run_ours(args, ws, rank, local):
                           "peak_source": peak_src},
         "route_compact_frac": round(route_frac, 4),
         "kernel_ms_per_step": {k: round(v[0] / prof_steps, 4) for k, v in prof.items()},
+        "kernel_gbs": {k: round(per_class_bytes[k] / (prof[k][0] / 1e3) / 1e9, 1)
+                       for k in per_class_bytes if prof[k][0] > 0},
         "e2e": {"value": round(ws * B * e2e_n / e2e_s, 2), "unit": "tokens/s",
                 "h2d_bytes_per_step": B * s.d_model * 4 + B * 4,
                 "d2h_bytes_per_step": B * s.d_model * 4 + B * s.n_layers},

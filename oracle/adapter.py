@@ -19,7 +19,10 @@ from . import buddy_oracle as O
 
 
 def to_f64(t: torch.Tensor) -> np.ndarray:
-    t = t.detach().to("cpu").contiguous()
+    """Exact float64 copy of a bf16 / fp32 tensor (converted where it lives)."""
+    if t.is_cuda:
+        return t.detach().to(torch.float64).cpu().numpy()
+    t = t.detach().contiguous()
     if t.dtype == torch.bfloat16:
         return O.bf16_bits_to_f64(t.view(torch.int16).numpy().view(np.uint16))
     if t.dtype == torch.float32:
@@ -74,6 +77,17 @@ def build_state(shape: ModelShape, seed: int, n_ctx: Sequence[int],
             V = to_f64(synth.kv_block(shape, seed, "v", l, i, 0, n, gen_device))
             st.set(l, i, K, V)
     return st
+
+
+def lazy_state(shape: ModelShape, seed: int, n_ctx: Sequence[int], gen_device: str = "cpu") -> O.KVState:
+    """KV state whose caches are generated on first use, one (layer, sequence)
+    at a time, and dropped by the oracle after each layer."""
+    def load(l, i):
+        n = int(n_ctx[i])
+        K = to_f64(synth.kv_block(shape, seed, "k", l, i, 0, n, gen_device))
+        V = to_f64(synth.kv_block(shape, seed, "v", l, i, 0, n, gen_device))
+        return K, V
+    return O.KVState(n_ctx, loader=load)
 
 
 def workload_inputs(w: Workload, step: int) -> np.ndarray:

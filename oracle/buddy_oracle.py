@@ -30,8 +30,13 @@ What it computes (plain numpy, float64 arithmetic, one sequence at a time):
 
 Precision.  The paper runs its model in bfloat16 (Sec. 5 "Hyper-parameters").
 For "bf16" shapes the oracle rounds exactly where a bf16 model stores a
-tensor: the normalised GEMM inputs, the K/V written to the cache, the
-attention output and the SwiGLU product (round-to-nearest-even through fp32).
+tensor: the K/V written to the cache and, in every layer but the first, the
+normalised GEMM inputs, the attention output and the SwiGLU product
+(round-to-nearest-even through fp32).  The first layer, whose output is the
+router's input, keeps its activations unrounded: rounding there makes the
+layer output jump by ~1e-3 when an input moves by ~1e-7 (a flipped bf16
+rounding of one element changes every SwiGLU product it feeds), and the
+routing decision would then not be a function of the mathematics.
 Everything else — projections, attention scores and softmax, residual
 stream, Decision Module — is float64.  "f32" shapes round nothing.
 
@@ -133,21 +138,31 @@ class Model:
 
 class KVState:
     """Per-(layer, sequence) caches.  kv[(l, i)] = (K, V), each [n, n_kv, hd]
-    float64 holding the stored values of positions 0..n-1."""
+    float64 holding the stored values of positions 0..n-1.  An optional
+    `loader(l, i)` supplies caches on first use (and `drop` forgets them), so
+    that large workloads can be evaluated one layer at a time."""
 
-    def __init__(self, n_ctx: Sequence[int]):
+    def __init__(self, n_ctx: Sequence[int], loader: Optional[Callable[[int, int], tuple]] = None):
         self.n = [int(v) for v in n_ctx]          # n_i: cached positions per sequence
         self.kv: Dict[tuple, tuple] = {}
+        self.loader = loader
 
     def set(self, layer: int, seq: int, K: np.ndarray, V: np.ndarray):
         assert K.shape[0] == self.n[seq] and V.shape == K.shape
         self.kv[(layer, seq)] = (np.asarray(K, np.float64), np.asarray(V, np.float64))
 
     def get(self, layer: int, seq: int):
+        if (layer, seq) not in self.kv and self.loader is not None:
+            K, V = self.loader(layer, seq)
+            self.set(layer, seq, K, V)
         return self.kv[(layer, seq)]
 
+    def drop(self, layer: int):
+        for key in [k for k in self.kv if k[0] == layer]:
+            del self.kv[key]
+
     def has(self, layer: int, seq: int) -> bool:
-        return (layer, seq) in self.kv
+        return (layer, seq) in self.kv or self.loader is not None
 
 
 # ---------------------------------------------------------------------------
@@ -193,11 +208,13 @@ def decode_attention(q: np.ndarray, K: np.ndarray, V: np.ndarray, group: int) ->
 
 
 def decoder_layer(sh: Shape, W: LayerWeights, h: np.ndarray, K_cache: np.ndarray,
-                  V_cache: np.ndarray, pos: int):
+                  V_cache: np.ndarray, pos: int, round_act: bool = True):
     """One executed block for one token at position `pos` = number of cached
-    positions.  Returns (h + F_l(h), K_t, V_t) with K_t, V_t [n_kv, hd] as stored."""
+    positions.  Returns (h + F_l(h), K_t, V_t) with K_t, V_t [n_kv, hd] as stored.
+    round_act=False keeps the GEMM inputs unrounded (the first layer)."""
     hd = sh.head_dim
-    xn = sh.store(rms_norm(h, W.attn_norm, sh.rms_eps))
+    act = sh.store if round_act else (lambda x: x)
+    xn = act(rms_norm(h, W.attn_norm, sh.rms_eps))
     q = W.w_q @ xn
     k = W.w_k @ xn
     v = W.w_v @ xn
@@ -209,10 +226,10 @@ def decoder_layer(sh: Shape, W: LayerWeights, h: np.ndarray, K_cache: np.ndarray
     v_t = sh.store(v.reshape(sh.n_kv_heads, hd))
     K = np.concatenate([K_cache, k_t[None]], axis=0)
     V = np.concatenate([V_cache, v_t[None]], axis=0)
-    attn = sh.store(decode_attention(q, K, V, sh.group).reshape(-1))
+    attn = act(decode_attention(q, K, V, sh.group).reshape(-1))
     h = h + W.w_o @ attn
-    xn2 = sh.store(rms_norm(h, W.ffn_norm, sh.rms_eps))
-    a = sh.store(silu(W.w_gate @ xn2) * (W.w_up @ xn2))
+    xn2 = act(rms_norm(h, W.ffn_norm, sh.rms_eps))
+    a = act(silu(W.w_gate @ xn2) * (W.w_up @ xn2))
     h = h + W.w_down @ a
     return h, k_t, v_t
 
@@ -289,7 +306,7 @@ def first_layer_and_route(model: Model, st: KVState, h_in: np.ndarray, k: Sequen
     kv0 = []
     for i in range(B):
         K, V = st.get(0, i)
-        h1[i], k_t, v_t = decoder_layer(sh, W0, h_in[i].astype(np.float64), K, V, st.n[i])
+        h1[i], k_t, v_t = decoder_layer(sh, W0, h_in[i].astype(np.float64), K, V, st.n[i], round_act=False)
         kv0.append((k_t, v_t))
     scores = np.empty((B, sh.l_mid))
     sel = []
@@ -341,6 +358,8 @@ def routed_layers(model: Model, st: KVState, route: RouteResult,
                 kv_new[(l, i)] = (k_t, v_t)
             else:
                 kv_new[(l, i)] = (zeros.copy(), zeros.copy())
+        if st.loader is not None:
+            st.drop(l)
     return StepResult(h, route.scores, route.sel, mask, rows, kv_new)
 
 
@@ -378,6 +397,6 @@ def dense_decode_step(model: Model, st: KVState, h_in: np.ndarray) -> Dict[int, 
         h = h_in[i].astype(np.float64)
         for l in range(sh.n_layers):
             K, V = st.get(l, i)
-            h, _, _ = decoder_layer(sh, model.layer(l), h, K, V, st.n[i])
+            h, _, _ = decoder_layer(sh, model.layer(l), h, K, V, st.n[i], round_act=(l != 0))
         out[i] = h
     return out

@@ -6,6 +6,7 @@
 
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <functional>
 #include <new>
@@ -53,8 +54,8 @@ static void free_ctx(buddy_ctx* x) {
   for (auto& kv : c.graphs) cudaGraphExecDestroy(kv.second);
   for (cudaEvent_t e : c.ev_pool) cudaEventDestroy(e);
   void* ptrs[] = {c.rope_cos, c.rope_sin, c.status, c.xn, c.act, c.attn_out, c.qkv, c.q,
-                  c.attn_m, c.attn_l, c.attn_acc, c.dm_u, c.mask, c.sel, c.scores, c.rows,
-                  c.count, c.h_in_stage, c.h_out_stage, c.k_stage, c.mask_stage, c.tmaps,
+                  c.attn_m, c.attn_l, c.attn_acc, c.attn_ctr, c.dm_u, c.mask, c.sel, c.scores, c.rows,
+                  c.count, c.h_in_stage, c.h_out_stage, c.k_stage, c.mask_stage, c.xn_lo, c.act_lo, c.attn_lo,
                   c.gemm_ws, c.gemm_ctr};
   for (void* p : ptrs)
     if (p) cudaFree(p);
@@ -106,6 +107,10 @@ extern "C" int buddy_create(const buddy_config* cfg, buddy_ctx** out) {
   c.qd = c.nq * c.hd; c.kvd = c.nkv * c.hd; c.qkvN = c.qd + 2 * c.kvd;
   c.maxB = g.max_batch; c.max_pos = g.max_pos; c.dtype = g.dtype;
   c.esz = g.dtype == BUDDY_DTYPE_BF16 ? 2 : 4;
+  {
+    const char* env = getenv("BUDDY_PDL");
+    c.pdl = !(env && env[0] == '0');
+  }
   auto fail = [&](cudaError_t e) {
     fprintf(stderr, "libbuddy: create: %s\n", cudaGetErrorString(e));
     free_ctx(x);
@@ -116,7 +121,7 @@ extern "C" int buddy_create(const buddy_config* cfg, buddy_ctx** out) {
   if ((e = cudaDeviceGetAttribute(&c.num_sms, cudaDevAttrMultiProcessorCount, c.device)) != cudaSuccess)
     return fail(e);
   const size_t B = c.maxB;
-  c.attn_chunk = 128;
+  c.attn_chunk = attention_chunk();
   c.attn_max_chunks = (c.max_pos + c.attn_chunk - 1) / c.attn_chunk;
   const size_t hmax = (size_t)c.max_pos * (c.hd / 2);
   if ((e = dalloc(&c.rope_cos, hmax)) || (e = dalloc(&c.rope_sin, hmax)) ||
@@ -127,13 +132,20 @@ extern "C" int buddy_create(const buddy_config* cfg, buddy_ctx** out) {
       (e = dalloc(&c.attn_m, B * c.nq * c.attn_max_chunks)) ||
       (e = dalloc(&c.attn_l, B * c.nq * c.attn_max_chunks)) ||
       (e = dalloc(&c.attn_acc, B * c.nq * c.attn_max_chunks * c.hd)) ||
+      (e = dalloc(&c.attn_ctr, B * c.nkv)) ||
       (e = dalloc(&c.dm_u, B * c.r)) || (e = dalloc(&c.mask, B * c.L)) ||
       (e = dalloc(&c.sel, B * c.Lm)) || (e = dalloc(&c.scores, B * c.Lm)) ||
       (e = dalloc(&c.rows, (size_t)c.L * B)) || (e = dalloc(&c.count, (size_t)c.L)) ||
       (e = dalloc(&c.h_in_stage, B * c.d)) || (e = dalloc(&c.h_out_stage, B * c.d)) ||
       (e = dalloc(&c.k_stage, B)) || (e = dalloc(&c.mask_stage, B * c.L)))
     return fail(e);
-  if ((e = cudaMemset(c.status, 0, 4 * sizeof(int32_t))) != cudaSuccess) return fail(e);
+  c.split0 = c.dtype == BUDDY_DTYPE_BF16;
+  if (c.split0 && ((e = cudaMalloc(&c.xn_lo, B * c.d * c.esz)) || (e = cudaMalloc(&c.act_lo, B * c.F * c.esz)) ||
+                   (e = cudaMalloc(&c.attn_lo, B * c.qd * c.esz))))
+    return fail(e);
+  if ((e = cudaMemset(c.status, 0, 4 * sizeof(int32_t))) != cudaSuccess ||
+      (e = cudaMemset(c.attn_ctr, 0, B * c.nkv * sizeof(int32_t))) != cudaSuccess)
+    return fail(e);
   if ((e = cudaStreamCreateWithFlags(&x->cap_stream, cudaStreamNonBlocking)) != cudaSuccess ||
       (e = cudaStreamCreateWithFlags(&x->body_stream, cudaStreamNonBlocking)) != cudaSuccess)
     return fail(e);
@@ -277,8 +289,9 @@ extern "C" int buddy_profile_read(buddy_ctx* ctx, int32_t n_cls, float* ms, int3
 // ---------------------------------------------------------------------------
 static void run_gemm(const Ctx& c, int epi, GemmArgs a, int layer, int which, cudaStream_t s) {
   a.status = c.status;
+  a.layer = layer;
+  a.which = which;
   if (c.use_tc) {
-    a.tmap_w = c.tmaps + (size_t)layer * 4 + which;
     launch_gemm_tc(c, epi, a, s);
   } else {
     launch_gemm_simt(c, epi, a, s);
@@ -291,14 +304,18 @@ static void run_gemm(const Ctx& c, int epi, GemmArgs a, int layer, int which, cu
 static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, const float* src,
                           float* H, cudaStream_t s, bool prof) {
   const buddy_layer_weights& W = c.layers[l];
+  // The first layer feeds the router: its GEMM inputs are kept as bf16 hi + lo
+  // pairs so that its output is a continuous function of the inputs.
+  const bool split = c.split0 && l == 0;
   {
     ProfScope p(c, s, BUDDY_PROF_RMSNORM, 1, prof);
-    launch_rmsnorm(c, src, sel, W.attn_norm, c.xn, s);
+    launch_rmsnorm(c, src, sel, W.attn_norm, c.xn, split ? c.xn_lo : nullptr, s);
   }
   GemmArgs g{};
   g.sel = sel;
   g.max_m = sel.n;
-  g.W = W.w_qkv; g.X = c.xn; g.N = c.qkvN; g.K = c.d; g.out_f32 = c.qkv;
+  g.split = split;
+  g.W = W.w_qkv; g.X = c.xn; g.X_lo = c.xn_lo; g.N = c.qkvN; g.K = c.d; g.out_f32 = c.qkv;
   {
     ProfScope p(c, s, BUDDY_PROF_GEMM_QKV, 1, prof);
     run_gemm(c, EPI_STORE_F32, g, l, 0, s);
@@ -309,29 +326,30 @@ static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, c
   }
   {
     ProfScope p(c, s, BUDDY_PROF_ATTENTION, 2, prof);
-    launch_attention(c, sel, kv, l, c.q, c.attn_out, s);
+    launch_attention(c, sel, kv, l, c.q, c.attn_out, split ? c.attn_lo : nullptr, s);
   }
   g = GemmArgs{};
-  g.sel = sel; g.max_m = sel.n;
-  g.W = W.w_o; g.X = c.attn_out; g.N = c.d; g.K = c.qd; g.resid_src = src; g.resid_dst = H;
+  g.sel = sel; g.max_m = sel.n; g.split = split;
+  g.W = W.w_o; g.X = c.attn_out; g.X_lo = c.attn_lo; g.N = c.d; g.K = c.qd; g.resid_src = src; g.resid_dst = H;
   {
     ProfScope p(c, s, BUDDY_PROF_GEMM_O, 1, prof);
     run_gemm(c, EPI_RESID, g, l, 1, s);
   }
   {
     ProfScope p(c, s, BUDDY_PROF_RMSNORM, 1, prof);
-    launch_rmsnorm(c, H, sel, W.ffn_norm, c.xn, s);
+    launch_rmsnorm(c, H, sel, W.ffn_norm, c.xn, split ? c.xn_lo : nullptr, s);
   }
   g = GemmArgs{};
-  g.sel = sel; g.max_m = sel.n;
-  g.W = W.w_gate_up; g.X = c.xn; g.N = c.F; g.K = c.d; g.out_act = c.act;
+  g.sel = sel; g.max_m = sel.n; g.split = split;
+  g.W = W.w_gate_up; g.X = c.xn; g.X_lo = c.xn_lo; g.N = c.F; g.K = c.d; g.out_act = c.act;
+  g.out_act_lo = split ? c.act_lo : nullptr;
   {
     ProfScope p(c, s, BUDDY_PROF_GEMM_GATE_UP, 1, prof);
     run_gemm(c, EPI_SWIGLU, g, l, 2, s);
   }
   g = GemmArgs{};
-  g.sel = sel; g.max_m = sel.n;
-  g.W = W.w_down; g.X = c.act; g.N = c.d; g.K = c.F; g.resid_src = H; g.resid_dst = H;
+  g.sel = sel; g.max_m = sel.n; g.split = split;
+  g.W = W.w_down; g.X = c.act; g.X_lo = c.act_lo; g.N = c.d; g.K = c.F; g.resid_src = H; g.resid_dst = H;
   {
     ProfScope p(c, s, BUDDY_PROF_GEMM_DOWN, 1, prof);
     run_gemm(c, EPI_RESID, g, l, 3, s);

@@ -51,6 +51,15 @@ __device__ __forceinline__ float warp_max(float v) {
 __device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x)); }
 
 // ---------------------------------------------------------------------------
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialisation may start while its predecessor runs; it must pass pdl_wait()
+// before reading anything an earlier kernel wrote.  pdl_trigger() lets the
+// next kernel start launching.  Both are no-ops for ordinary launches.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// ---------------------------------------------------------------------------
 // Per-call device status: status[0] sticky error bits, status[1] abort flag of
 // the call in flight (set by the call's first kernel, read by all others).
 // ---------------------------------------------------------------------------

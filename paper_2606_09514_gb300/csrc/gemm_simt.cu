@@ -14,12 +14,15 @@ constexpr int kSimtRows = 4;
 
 template <typename T, int EPI>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ W,
-                                                        const T* __restrict__ X, int N, int K,
+                                                        const T* __restrict__ X, const T* __restrict__ X_lo,
+                                                        int N, int K,
                                                         const int32_t* rows, const int32_t* count,
                                                         int n, float* __restrict__ out_f32,
-                                                        T* __restrict__ out_act,
+                                                        T* __restrict__ out_act, T* __restrict__ out_act_lo,
                                                         const float* resid_src, float* resid_dst,
                                                         const int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
   if (call_aborted(status)) return;
   const int m = count ? *count : n;
   const int unit = blockIdx.x * 8 + (threadIdx.x >> 5);
@@ -44,6 +47,12 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ W,
         if (j0 + r < m) {
           float xv[8];
           load8(X + (size_t)(j0 + r) * K + k, xv);
+          if (X_lo) {
+            float xl[8];
+            load8(X_lo + (size_t)(j0 + r) * K + k, xl);
+#pragma unroll
+            for (int u = 0; u < 8; ++u) xv[u] += xl[u];
+          }
 #pragma unroll
           for (int a = 0; a < NR; ++a)
 #pragma unroll
@@ -70,38 +79,42 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ W,
         const int i = rows ? rows[j] : j;
         resid_dst[(size_t)i * N + unit] = resid_src[(size_t)i * N + unit] + v0;
       } else {
-        out_act[(size_t)j * N + unit] = from_f<T>(silu_f(v0) * v1);
+        const float a = silu_f(v0) * v1;
+        const T hi = from_f<T>(a);
+        out_act[(size_t)j * N + unit] = hi;
+        if (out_act_lo) out_act_lo[(size_t)j * N + unit] = from_f<T>(a - to_f(hi));
       }
     }
   }
 }
 
 template <typename T>
-static void simt_dispatch(int epi, const GemmArgs& a, cudaStream_t s) {
+static void simt_dispatch(int epi, const GemmArgs& a, cudaStream_t s, bool pdl) {
   const unsigned grid = (unsigned)((a.N + 7) / 8);
   const T* W = (const T*)a.W;
   const T* X = (const T*)a.X;
+  const T* Xl = a.split ? (const T*)a.X_lo : nullptr;
   switch (epi) {
     case EPI_STORE_F32:
-      gemm_simt_kernel<T, EPI_STORE_F32><<<grid, 256, 0, s>>>(W, X, a.N, a.K, a.sel.rows, a.sel.count,
-                                                              a.sel.n, a.out_f32, nullptr, nullptr,
-                                                              nullptr, a.status);
+      launch_k(gemm_simt_kernel<T, EPI_STORE_F32>, grid, 256, 0, s, pdl, W, X, Xl, a.N, a.K, a.sel.rows,
+               a.sel.count, a.sel.n, a.out_f32, (T*)nullptr, (T*)nullptr, (const float*)nullptr, (float*)nullptr,
+               a.status);
       break;
     case EPI_RESID:
-      gemm_simt_kernel<T, EPI_RESID><<<grid, 256, 0, s>>>(W, X, a.N, a.K, a.sel.rows, a.sel.count,
-                                                          a.sel.n, nullptr, nullptr, a.resid_src,
-                                                          a.resid_dst, a.status);
+      launch_k(gemm_simt_kernel<T, EPI_RESID>, grid, 256, 0, s, pdl, W, X, Xl, a.N, a.K, a.sel.rows,
+               a.sel.count, a.sel.n, (float*)nullptr, (T*)nullptr, (T*)nullptr, a.resid_src, a.resid_dst,
+               a.status);
       break;
     default:
-      gemm_simt_kernel<T, EPI_SWIGLU><<<grid, 256, 0, s>>>(W, X, a.N, a.K, a.sel.rows, a.sel.count,
-                                                           a.sel.n, nullptr, (T*)a.out_act, nullptr,
-                                                           nullptr, a.status);
+      launch_k(gemm_simt_kernel<T, EPI_SWIGLU>, grid, 256, 0, s, pdl, W, X, Xl, a.N, a.K, a.sel.rows,
+               a.sel.count, a.sel.n, (float*)nullptr, (T*)a.out_act, (T*)a.out_act_lo, (const float*)nullptr,
+               (float*)nullptr, a.status);
   }
 }
 
 void launch_gemm_simt(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s) {
-  if (c.dtype == BUDDY_DTYPE_BF16) simt_dispatch<bf16>(epi, a, s);
-  else simt_dispatch<float>(epi, a, s);
+  if (c.dtype == BUDDY_DTYPE_BF16) simt_dispatch<bf16>(epi, a, s, c.pdl);
+  else simt_dispatch<float>(epi, a, s, c.pdl);
 }
 
 }  // namespace buddy

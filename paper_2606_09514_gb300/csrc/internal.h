@@ -6,6 +6,7 @@
 #include <stdint.h>
 
 #include <map>
+#include <utility>
 #include <vector>
 
 #include "../../include/buddy.h"
@@ -41,18 +42,36 @@ struct GemmArgs {
   // epilogues
   float* out_f32;         // EPI_STORE_F32: [m, N]
   void* out_act;          // EPI_SWIGLU: [m, N] act dtype
+  void* X_lo;             // split activations: bf16 remainder of X (or null)
+  void* out_act_lo;       // split activations: bf16 remainder of the SwiGLU output
+  bool split;
   const float* resid_src; // EPI_RESID: dst[i] = src[i] + acc  (may equal dst)
   float* resid_dst;
   const int32_t* status;
-  // tcgen05 path: tensor maps (device-side copies live in the context)
-  const CUtensorMap* tmap_w;
-  const CUtensorMap* tmap_x;
-  int splits;             // split-K factor chosen by the host
-  float* ws;              // split-K partial workspace
-  int32_t* tile_ctr;      // split-K arrival counters (self-resetting)
+  int layer;              // tensor-core path: which layer's weight map
+  int which;              // 0 qkv, 1 o, 2 gate_up, 3 down
 };
 
 struct Ctx;
+
+// Launch with programmatic stream serialisation when `pdl` is set (the kernel
+// then overlaps its prologue with the predecessor and synchronises with
+// pdl_wait()).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                            bool pdl, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = pdl ? attr : nullptr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
 
 // Kernel launchers (kernels.cu)
 void launch_rope_table(float* cos_t, float* sin_t, int max_pos, int hd, double theta, cudaStream_t s);
@@ -60,13 +79,14 @@ void launch_step_check(const Ctx& c, int B, const int32_t* k, const int32_t* len
                        int extra_pos, int32_t* status, cudaStream_t s);
 void launch_kv_check(const Ctx& c, int n_seq, const int32_t* seq_ids, int n_new, int batch,
                      const int32_t* len, const int32_t* cap, int32_t* status, cudaStream_t s);
-void launch_rmsnorm(const Ctx& c, const float* H, RowSel sel, const float* gamma, void* xn,
+void launch_rmsnorm(const Ctx& c, const float* H, RowSel sel, const float* gamma, void* xn, void* xn_lo,
                     cudaStream_t s);
 void launch_qkv_finalize(const Ctx& c, const float* qkv, const float* bias, RowSel sel,
                          const buddy_kv_state& kv, int layer, float* q_out, float* pool,
                          cudaStream_t s);
 void launch_attention(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q,
-                      void* attn_out, cudaStream_t s);
+                      void* attn_out, void* attn_lo, cudaStream_t s);   // attention.cu
+int attention_chunk();
 void launch_route(const Ctx& c, int B, const float* h1, const float* pool, const int32_t* len,
                   int len_bias, const int32_t* k, uint8_t* mask, int32_t* sel, float* scores,
                   cudaStream_t s);
@@ -92,6 +112,7 @@ struct Ctx {
   int dtype;
   size_t esz;
   int device, num_sms;
+  bool pdl = true;             // programmatic dependent launch between step kernels
 
   bool have_weights = false;
   std::vector<buddy_layer_weights> layers;
@@ -104,12 +125,18 @@ struct Ctx {
   void* xn = nullptr;          // [maxB, d]   act dtype: normalised GEMM input
   void* act = nullptr;         // [maxB, F]   act dtype: SwiGLU output
   void* attn_out = nullptr;    // [maxB, qd]  act dtype
+  // first layer (the router's input) keeps activations as bf16 hi + lo pairs
+  bool split0 = false;
+  void* xn_lo = nullptr;       // [maxB, d]
+  void* act_lo = nullptr;      // [maxB, F]
+  void* attn_lo = nullptr;     // [maxB, qd]
   float* qkv = nullptr;        // [maxB, qkvN]
   float* q = nullptr;          // [maxB, qd]
   int attn_chunk = 128, attn_max_chunks = 1;
   float* attn_m = nullptr;     // [maxB, nq, max_chunks]
   float* attn_l = nullptr;
   float* attn_acc = nullptr;   // [maxB, nq, max_chunks, hd]
+  int32_t* attn_ctr = nullptr; // [maxB, nkv] chunk arrivals (self-resetting)
   float* dm_u = nullptr;       // [maxB, r]
   uint8_t* mask = nullptr;     // [maxB, L]
   int32_t* sel = nullptr;      // [maxB, Lm]
@@ -124,8 +151,10 @@ struct Ctx {
 
   // tcgen05 GEMM resources
   bool use_tc = false;
-  CUtensorMap* tmaps = nullptr;           // device array: per layer 4 weight maps + 3 activation maps
-  std::vector<CUtensorMap> tmaps_host;
+  std::vector<CUtensorMap> tmaps_host;    // per layer 4 weight maps, then 3 activation maps
+  int tc_bn_max = 16, tc_stages[2] = {1, 1}, tc_smem[2] = {0, 0};   // [plain, split activations]
+  uint32_t tc_stage_bytes[2] = {0, 0}, tc_tmem_cols = 32;
+  int tc_splits[4] = {1, 1, 1, 1}, tc_tiles[4] = {1, 1, 1, 1};
   float* gemm_ws = nullptr;
   size_t gemm_ws_elems = 0;
   int32_t* gemm_ctr = nullptr;

@@ -1,6 +1,5 @@
 // Non-GEMM kernels of the budget-routed decode step: argument checks, RMSNorm,
-// QKV finalisation (bias, RoPE, cache append, pooled-context update), split-K
-// decode attention, the router (KV-aware pooling + Decision Module + top-k),
+// QKV finalisation (bias, RoPE, cache append, pooled-context update), the router (KV-aware pooling + Decision Module + top-k),
 // row compaction with zero K/V for skipped layers, and KV prefill.
 #include <cuda_runtime.h>
 
@@ -33,6 +32,8 @@ void launch_rope_table(float* c, float* s, int max_pos, int hd, double theta, cu
 // ---------------------------------------------------------------------------
 __global__ void step_check_kernel(int B, const int32_t* k, int Lm, const int32_t* len,
                                   const int32_t* cap, int extra, int max_pos, int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ int bad;
   if (threadIdx.x == 0) bad = 0;
   __syncthreads();
@@ -55,11 +56,13 @@ __global__ void step_check_kernel(int B, const int32_t* k, int Lm, const int32_t
 
 void launch_step_check(const Ctx& c, int B, const int32_t* k, const int32_t* len, const int32_t* cap,
                        int extra, int32_t* status, cudaStream_t s) {
-  step_check_kernel<<<1, 256, 0, s>>>(B, k, c.Lm, len, cap, extra, c.max_pos, status);
+  launch_k(step_check_kernel, 1, 256, 0, s, c.pdl, B, k, c.Lm, len, cap, extra, c.max_pos, status);
 }
 
 __global__ void kv_check_kernel(int n_seq, const int32_t* ids, int n_new, int batch,
                                 const int32_t* len, const int32_t* cap, int max_pos, int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ int bad;
   if (threadIdx.x == 0) bad = 0;
   __syncthreads();
@@ -83,7 +86,7 @@ __global__ void kv_check_kernel(int n_seq, const int32_t* ids, int n_new, int ba
 
 void launch_kv_check(const Ctx& c, int n_seq, const int32_t* ids, int n_new, int batch,
                      const int32_t* len, const int32_t* cap, int32_t* status, cudaStream_t s) {
-  kv_check_kernel<<<1, 256, 0, s>>>(n_seq, ids, n_new, batch, len, cap, c.max_pos, status);
+  launch_k(kv_check_kernel, 1, 256, 0, s, c.pdl, n_seq, ids, n_new, batch, len, cap, c.max_pos, status);
 }
 
 // ---------------------------------------------------------------------------
@@ -107,7 +110,10 @@ template <typename T>
 __global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ H, int d,
                                                       const int32_t* rows, const int32_t* count, int n,
                                                       const float* __restrict__ gamma, float eps,
-                                                      T* __restrict__ xn, const int32_t* status) {
+                                                      T* __restrict__ xn, T* __restrict__ xn_lo,
+                                                      const int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
   if (call_aborted(status)) return;
   const int m = count ? *count : n;
   const int j = blockIdx.x;
@@ -123,24 +129,28 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ 
   ss = block_sum_256(ss, red);
   const float inv = rsqrtf(ss / (float)d + eps);
   T* o = xn + (size_t)j * d;
+  T* olo = xn_lo ? xn_lo + (size_t)j * d : nullptr;
   for (int e = threadIdx.x * 4; e < d; e += blockDim.x * 4) {
     const float4 v = *reinterpret_cast<const float4*>(h + e);
     const float4 g = *reinterpret_cast<const float4*>(gamma + e);
-    o[e + 0] = from_f<T>(v.x * inv * g.x);
-    o[e + 1] = from_f<T>(v.y * inv * g.y);
-    o[e + 2] = from_f<T>(v.z * inv * g.z);
-    o[e + 3] = from_f<T>(v.w * inv * g.w);
+    const float y[4] = {v.x * inv * g.x, v.y * inv * g.y, v.z * inv * g.z, v.w * inv * g.w};
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const T hi = from_f<T>(y[u]);
+      o[e + u] = hi;
+      if (olo) olo[e + u] = from_f<T>(y[u] - to_f(hi));   // remainder term (split activations)
+    }
   }
 }
 
-void launch_rmsnorm(const Ctx& c, const float* H, RowSel sel, const float* gamma, void* xn,
+void launch_rmsnorm(const Ctx& c, const float* H, RowSel sel, const float* gamma, void* xn, void* xn_lo,
                     cudaStream_t s) {
   if (c.dtype == BUDDY_DTYPE_BF16)
-    rmsnorm_kernel<bf16><<<sel.n, 256, 0, s>>>(H, c.d, sel.rows, sel.count, sel.n, gamma,
-                                               c.cfg.rms_eps, (bf16*)xn, c.status);
+    launch_k(rmsnorm_kernel<bf16>, sel.n, 256, 0, s, c.pdl, H, c.d, sel.rows, sel.count, sel.n, gamma,
+             c.cfg.rms_eps, (bf16*)xn, (bf16*)xn_lo, (const int32_t*)c.status);
   else
-    rmsnorm_kernel<float><<<sel.n, 256, 0, s>>>(H, c.d, sel.rows, sel.count, sel.n, gamma,
-                                                c.cfg.rms_eps, (float*)xn, c.status);
+    launch_k(rmsnorm_kernel<float>, sel.n, 256, 0, s, c.pdl, H, c.d, sel.rows, sel.count, sel.n, gamma,
+             c.cfg.rms_eps, (float*)xn, (float*)nullptr, (const int32_t*)c.status);
 }
 
 // ---------------------------------------------------------------------------
@@ -154,6 +164,8 @@ __global__ void __launch_bounds__(256) qkv_finalize_kernel(
     const int32_t* count, int n, int nq, int nkv, int hd, const float* __restrict__ rc,
     const float* __restrict__ rs, const int32_t* len, const int64_t* seq_off, const int32_t* cap,
     T* Kc, T* Vc, float* __restrict__ q_out, float* pool, const int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
   if (call_aborted(status)) return;
   const int m = count ? *count : n;
   const int j = blockIdx.x;
@@ -201,159 +213,15 @@ void launch_qkv_finalize(const Ctx& c, const float* qkv, const float* bias, RowS
                          const buddy_kv_state& kv, int layer, float* q_out, float* pool,
                          cudaStream_t s) {
   if (c.dtype == BUDDY_DTYPE_BF16)
-    qkv_finalize_kernel<bf16><<<sel.n, 256, 0, s>>>(
-        qkv, bias, sel.rows, sel.count, sel.n, c.nq, c.nkv, c.hd, c.rope_cos, c.rope_sin, kv.len,
-        kv.seq_off, kv.cap, (bf16*)kv.k_cache[layer], (bf16*)kv.v_cache[layer], q_out, pool, c.status);
+    launch_k(qkv_finalize_kernel<bf16>, sel.n, 256, 0, s, c.pdl,
+             qkv, bias, sel.rows, sel.count, sel.n, c.nq, c.nkv, c.hd, (const float*)c.rope_cos,
+             (const float*)c.rope_sin, (const int32_t*)kv.len, kv.seq_off, kv.cap, (bf16*)kv.k_cache[layer],
+             (bf16*)kv.v_cache[layer], q_out, pool, (const int32_t*)c.status);
   else
-    qkv_finalize_kernel<float><<<sel.n, 256, 0, s>>>(
-        qkv, bias, sel.rows, sel.count, sel.n, c.nq, c.nkv, c.hd, c.rope_cos, c.rope_sin, kv.len,
-        kv.seq_off, kv.cap, (float*)kv.k_cache[layer], (float*)kv.v_cache[layer], q_out, pool,
-        c.status);
-}
-
-// ---------------------------------------------------------------------------
-// Decode attention (Eq. 9) for one layer, split over KV chunks.
-// CTA = (chunk, kv head g, active row j), HD threads.  All G = n_q/n_kv query
-// heads of the group share one pass over the chunk's K and V.  Positions
-// 0..len[i] (the new token included) are attended; zero-filled positions of
-// skipped steps take part with logit 0 (Sec. 6).
-// Partials (running max, sum of exponentials, unnormalised output) per chunk,
-// merged by attn_combine_kernel.
-// ---------------------------------------------------------------------------
-constexpr int kMaxGroup = 8;
-
-template <typename T, int HD>
-__global__ void __launch_bounds__(HD) attn_partial_kernel(
-    const float* __restrict__ q, const int32_t* rows, const int32_t* count, int n, int nq, int nkv,
-    const int32_t* len, const int64_t* seq_off, const int32_t* cap, const T* __restrict__ Kc,
-    const T* __restrict__ Vc, int chunk, int max_chunks, float* __restrict__ part_m,
-    float* __restrict__ part_l, float* __restrict__ part_acc, const int32_t* status) {
-  if (call_aborted(status)) return;
-  const int m = count ? *count : n;
-  const int c = blockIdx.x, g = blockIdx.y, j = blockIdx.z;
-  if (j >= m) return;
-  const int i = rows ? rows[j] : j;
-  const int npos = len[i] + 1;
-  const int p0 = c * chunk;
-  if (p0 >= npos) return;
-  const int p1 = min(npos, p0 + chunk);
-  const int G = nq / nkv;
-  constexpr int NW = HD / 32;
-  constexpr int EPL = HD / 32;  // channels per lane
-  extern __shared__ float sm[];
-  float* qs = sm;                   // [G][HD]
-  float* ss = sm + G * HD;          // [G][chunk]
-  __shared__ float mx_s[kMaxGroup], sum_s[kMaxGroup];
-  const float scale = rsqrtf((float)HD);
-  for (int t = threadIdx.x; t < G * HD; t += HD)
-    qs[t] = q[(size_t)j * nq * HD + (size_t)g * G * HD + t] * scale;
-  __syncthreads();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const T* Kb = Kc + kv_offset(seq_off, cap, i, nkv, HD, g, 0);
-  const T* Vb = Vc + kv_offset(seq_off, cap, i, nkv, HD, g, 0);
-  // logits
-  for (int p = p0 + warp; p < p1; p += NW) {
-    float kv[EPL];
-#pragma unroll
-    for (int u = 0; u < EPL; ++u) kv[u] = to_f(Kb[(size_t)p * HD + lane * EPL + u]);
-    for (int h = 0; h < G; ++h) {
-      float a = 0.f;
-#pragma unroll
-      for (int u = 0; u < EPL; ++u) a += qs[h * HD + lane * EPL + u] * kv[u];
-      a = warp_sum(a);
-      if (lane == 0) ss[h * chunk + (p - p0)] = a;
-    }
-  }
-  __syncthreads();
-  // per-head max and exponentials
-  const int cnt = p1 - p0;
-  for (int h = warp; h < G; h += NW) {
-    float mxv = -INFINITY;
-    for (int t = lane; t < cnt; t += 32) mxv = fmaxf(mxv, ss[h * chunk + t]);
-    mxv = warp_max(mxv);
-    float sv = 0.f;
-    for (int t = lane; t < cnt; t += 32) {
-      const float e = expf(ss[h * chunk + t] - mxv);
-      ss[h * chunk + t] = e;
-      sv += e;
-    }
-    sv = warp_sum(sv);
-    if (lane == 0) {
-      mx_s[h] = mxv;
-      sum_s[h] = sv;
-    }
-  }
-  __syncthreads();
-  // P.V
-  const int e = threadIdx.x;
-  float acc[kMaxGroup];
-#pragma unroll
-  for (int h = 0; h < kMaxGroup; ++h) acc[h] = 0.f;
-  for (int p = p0; p < p1; ++p) {
-    const float v = to_f(Vb[(size_t)p * HD + e]);
-#pragma unroll
-    for (int h = 0; h < kMaxGroup; ++h)
-      if (h < G) acc[h] += ss[h * chunk + (p - p0)] * v;
-  }
-  for (int h = 0; h < G; ++h) {
-    const size_t slot = ((size_t)j * nq + g * G + h) * max_chunks + c;
-    part_acc[slot * HD + e] = acc[h];
-    if (e == 0) {
-      part_m[slot] = mx_s[h];
-      part_l[slot] = sum_s[h];
-    }
-  }
-}
-
-template <typename T, int HD>
-__global__ void __launch_bounds__(HD) attn_combine_kernel(
-    const int32_t* rows, const int32_t* count, int n, int nq, const int32_t* len, int chunk,
-    int max_chunks, const float* __restrict__ part_m, const float* __restrict__ part_l,
-    const float* __restrict__ part_acc, T* __restrict__ out, const int32_t* status) {
-  if (call_aborted(status)) return;
-  const int m = count ? *count : n;
-  const int j = blockIdx.x, h = blockIdx.y;
-  if (j >= m) return;
-  const int i = rows ? rows[j] : j;
-  const int nc = (len[i] + 1 + chunk - 1) / chunk;
-  const size_t base = ((size_t)j * nq + h) * max_chunks;
-  float M = -INFINITY;
-  for (int c = 0; c < nc; ++c) M = fmaxf(M, part_m[base + c]);
-  float Ls = 0.f, a = 0.f;
-  const int e = threadIdx.x;
-  for (int c = 0; c < nc; ++c) {
-    const float w = expf(part_m[base + c] - M);
-    Ls += part_l[base + c] * w;
-    a += part_acc[(base + c) * HD + e] * w;
-  }
-  out[(size_t)j * nq * HD + (size_t)h * HD + e] = from_f<T>(a / Ls);
-}
-
-template <typename T, int HD>
-static void attention_impl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer,
-                           const float* q, void* out, cudaStream_t s) {
-  const int G = c.nq / c.nkv;
-  dim3 grid(c.attn_max_chunks, c.nkv, sel.n);
-  const size_t smem = (size_t)G * (HD + c.attn_chunk) * sizeof(float);
-  attn_partial_kernel<T, HD><<<grid, HD, smem, s>>>(
-      q, sel.rows, sel.count, sel.n, c.nq, c.nkv, kv.len, kv.seq_off, kv.cap,
-      (const T*)kv.k_cache[layer], (const T*)kv.v_cache[layer], c.attn_chunk, c.attn_max_chunks,
-      c.attn_m, c.attn_l, c.attn_acc, c.status);
-  dim3 g2(sel.n, c.nq);
-  attn_combine_kernel<T, HD><<<g2, HD, 0, s>>>(sel.rows, sel.count, sel.n, c.nq, kv.len,
-                                               c.attn_chunk, c.attn_max_chunks, c.attn_m, c.attn_l,
-                                               c.attn_acc, (T*)out, c.status);
-}
-
-void launch_attention(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q,
-                      void* out, cudaStream_t s) {
-  if (c.dtype == BUDDY_DTYPE_BF16) {
-    if (c.hd == 128) attention_impl<bf16, 128>(c, sel, kv, layer, q, out, s);
-    else attention_impl<bf16, 64>(c, sel, kv, layer, q, out, s);
-  } else {
-    if (c.hd == 128) attention_impl<float, 128>(c, sel, kv, layer, q, out, s);
-    else attention_impl<float, 64>(c, sel, kv, layer, q, out, s);
-  }
+    launch_k(qkv_finalize_kernel<float>, sel.n, 256, 0, s, c.pdl,
+             qkv, bias, sel.rows, sel.count, sel.n, c.nq, c.nkv, c.hd, (const float*)c.rope_cos,
+             (const float*)c.rope_sin, (const int32_t*)kv.len, kv.seq_off, kv.cap, (float*)kv.k_cache[layer],
+             (float*)kv.v_cache[layer], q_out, pool, (const int32_t*)c.status);
 }
 
 // ---------------------------------------------------------------------------
@@ -368,6 +236,8 @@ __global__ void __launch_bounds__(256) route_hidden_kernel(
     int B, int d, int hd, int group, int nkv, const float* __restrict__ h1,
     const float* __restrict__ pool, const int32_t* len, int len_bias, const float* __restrict__ w1,
     const float* __restrict__ b1, int r, float* __restrict__ u, const int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
   if (call_aborted(status)) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int unit = blockIdx.x * 8 + warp;
@@ -424,6 +294,8 @@ __global__ void __launch_bounds__(64) route_select_kernel(
     int Lm, int r, const float* __restrict__ u, const float* __restrict__ w2,
     const float* __restrict__ b2, const float* __restrict__ prior, float omega, const int32_t* k,
     uint8_t* mask, int32_t* sel, float* scores, const int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
   if (call_aborted(status)) return;
   const int i = blockIdx.x;
   extern __shared__ float s[];           // [Lm]
@@ -467,11 +339,10 @@ void launch_route(const Ctx& c, int B, const float* h1, const float* pool, const
                   int len_bias, const int32_t* k, uint8_t* mask, int32_t* sel, float* scores,
                   cudaStream_t s) {
   dim3 g1((c.r + 7) / 8, (B + kRouteRows - 1) / kRouteRows);
-  route_hidden_kernel<<<g1, 256, 0, s>>>(B, c.d, c.hd, c.nq / c.nkv, c.nkv, h1, pool, len, len_bias,
-                                         c.dm.w1, c.dm.b1, c.r, c.dm_u, c.status);
-  route_select_kernel<<<B, 64, c.Lm * sizeof(float), s>>>(c.Lm, c.r, c.dm_u, c.dm.w2, c.dm.b2,
-                                                          c.dm.prior, c.dm.omega, k, mask, sel,
-                                                          scores, c.status);
+  launch_k(route_hidden_kernel, g1, 256, 0, s, c.pdl, B, c.d, c.hd, c.nq / c.nkv, c.nkv, h1, pool, len,
+           len_bias, c.dm.w1, c.dm.b1, c.r, c.dm_u, (const int32_t*)c.status);
+  launch_k(route_select_kernel, B, 64, c.Lm * sizeof(float), s, c.pdl, c.Lm, c.r, (const float*)c.dm_u,
+           c.dm.w2, c.dm.b2, c.dm.prior, c.dm.omega, k, mask, sel, scores, (const int32_t*)c.status);
 }
 
 // ---------------------------------------------------------------------------
@@ -487,6 +358,8 @@ __global__ void __launch_bounds__(1024) compact_kernel(int B, int L, int nkv, in
                                                        const int64_t* seq_off, const int32_t* cap,
                                                        int32_t* rows, int32_t* count,
                                                        const int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
   if (call_aborted(status)) return;
   const int l = blockIdx.x;
   int32_t* rl = rows + (size_t)l * B;
@@ -539,11 +412,11 @@ void launch_compact(const Ctx& c, int B, const uint8_t* mask, const buddy_kv_sta
     p.v[l] = kv.v_cache[l];
   }
   if (c.dtype == BUDDY_DTYPE_BF16)
-    compact_kernel<bf16><<<c.L, 1024, 0, s>>>(B, c.L, c.nkv, c.hd, mask, p, kv.len, kv.seq_off,
-                                              kv.cap, rows, count, c.status);
+    launch_k(compact_kernel<bf16>, c.L, 1024, 0, s, c.pdl, B, c.L, c.nkv, c.hd, mask, p,
+             (const int32_t*)kv.len, kv.seq_off, kv.cap, rows, count, (const int32_t*)c.status);
   else
-    compact_kernel<float><<<c.L, 1024, 0, s>>>(B, c.L, c.nkv, c.hd, mask, p, kv.len, kv.seq_off,
-                                               kv.cap, rows, count, c.status);
+    launch_k(compact_kernel<float>, c.L, 1024, 0, s, c.pdl, B, c.L, c.nkv, c.hd, mask, p,
+             (const int32_t*)kv.len, kv.seq_off, kv.cap, rows, count, (const int32_t*)c.status);
 }
 
 // ---------------------------------------------------------------------------
@@ -551,6 +424,8 @@ void launch_compact(const Ctx& c, int B, const uint8_t* mask, const buddy_kv_sta
 // ---------------------------------------------------------------------------
 __global__ void advance_kernel(int B, int32_t* len, int by, const int32_t* ids,
                                const int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
   if (call_aborted(status)) return;
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= B) return;
@@ -559,7 +434,7 @@ __global__ void advance_kernel(int B, int32_t* len, int by, const int32_t* ids,
 }
 
 void launch_advance(const Ctx& c, int B, int32_t* len, int by, const int32_t* ids, cudaStream_t s) {
-  advance_kernel<<<(B + 255) / 256, 256, 0, s>>>(B, len, by, ids, c.status);
+  launch_k(advance_kernel, (B + 255) / 256, 256, 0, s, c.pdl, B, len, by, ids, (const int32_t*)c.status);
 }
 
 // ---------------------------------------------------------------------------
@@ -573,6 +448,8 @@ __global__ void __launch_bounds__(256) kv_append_kernel(int n_new, int nkv, int 
                                                         const T* __restrict__ kn,
                                                         const T* __restrict__ vn, T* Kc, T* Vc,
                                                         const int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
   if (call_aborted(status)) return;
   const int t = blockIdx.x, jj = blockIdx.y;
   const int s = ids[jj];
@@ -593,6 +470,8 @@ __global__ void __launch_bounds__(256) pool_refresh_kernel(int n_new, int nkv, i
                                                            const int64_t* seq_off,
                                                            const int32_t* cap, const T* V0,
                                                            float* pool, const int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
   if (call_aborted(status)) return;
   const int s = ids[blockIdx.y];
   const int kvd = nkv * hd;

@@ -17,6 +17,9 @@ import numpy as np
 
 ROUTE_MARGIN = 1e-3
 HIDDEN_TOL = {"f32": 1e-4, "bf16": 2e-2}
+# K/V written at the new position derive from the same layer's hidden state:
+# same normwise-by-max bound
+KV_TOL = HIDDEN_TOL
 
 
 def adopt_routes(o_scores: np.ndarray, o_sel: Sequence[Sequence[int]], g_sel: Sequence[Sequence[int]],

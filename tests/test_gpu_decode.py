@@ -88,7 +88,7 @@ def run_parity(w, steps=None, use_graph=False, prior=False, check_kv=True):
                     gv = dw.kv.view("v", l, i)[:, pos, :].float().cpu().numpy()
                     ok, ov = res.kv_new[(l, i)]
                     if g_mask[i, l]:
-                        assert P.max_rel_err(gk, ok) < 2 * 2.0 ** -8 and P.max_rel_err(gv, ov) < 2 * 2.0 ** -8
+                        assert P.max_rel_err(gk, ok) < P.KV_TOL[s.dtype] and P.max_rel_err(gv, ov) < P.KV_TOL[s.dtype]
                     else:
                         assert not gk.any() and not gv.any()
     # positions advanced by one per step

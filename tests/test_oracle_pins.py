@@ -232,6 +232,28 @@ def test_decoder_layer_bf16_rounds_only_stored_tensors():
     assert 1e-6 < err < 2e-2
 
 
+def test_first_layer_keeps_activations_unrounded():
+    """round_act=False rounds only the stored K/V: with the same stored K/V the
+    bf16 layer equals the unrounded (f32-shape) layer."""
+    rng = np.random.default_rng(11)
+    sh32, sh16 = _tiny_shape(), _tiny_shape(dtype="bf16")
+    W = _rand_layer(sh32, rng)
+    K, V = rng.standard_normal((5, 2, 8)), rng.standard_normal((5, 2, 8))
+    h = rng.standard_normal(sh32.d_model)
+    b, kb, vb = O.decoder_layer(sh16, W, h, K, V, 5, round_act=False)
+    np.testing.assert_array_equal(O.round_to_bf16(kb), kb)
+    # recompute the f32 layer with the same (rounded) new K/V appended
+    xn = O.rms_norm(h, W.attn_norm, sh32.rms_eps)
+    q = O.rope((W.w_q @ xn + W.b_q).reshape(4, 8), 5, sh32.rope_theta)
+    att = O.decode_attention(q, np.concatenate([K, kb[None]]), np.concatenate([V, vb[None]]), 2).reshape(-1)
+    x = h + W.w_o @ att
+    xn2 = O.rms_norm(x, W.ffn_norm, sh32.rms_eps)
+    ref = x + W.w_down @ (O.silu(W.w_gate @ xn2) * (W.w_up @ xn2))
+    np.testing.assert_allclose(b, ref, rtol=1e-12, atol=1e-12)
+    a, _, _ = O.decoder_layer(sh16, W, h, K, V, 5, round_act=True)
+    assert np.max(np.abs(a - b)) > 0
+
+
 def test_dm_matches_torch_mlp():
     rng = np.random.default_rng(8)
     d2, r, Lm = 24, 10, 7
@@ -336,7 +358,7 @@ def test_skipped_layers_are_identity_and_store_zero_kv():
         st_ref = A.build_state(w.shape, w.seed, w.contexts(), seqs=[i])
         for l in [0] + res.sel[i] + [sh.n_layers - 1]:
             K, V = st_ref.get(l, i)
-            x, _, _ = O.decoder_layer(sh, model.layer(l), x, K, V, n0[i])
+            x, _, _ = O.decoder_layer(sh, model.layer(l), x, K, V, n0[i], round_act=(l != 0))
         np.testing.assert_array_equal(res.h_out[i], x)
         for l in range(sh.n_layers):
             K, V = st.get(l, i)
