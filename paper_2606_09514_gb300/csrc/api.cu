@@ -316,13 +316,20 @@ static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, c
   g.max_m = sel.n;
   g.split = split;
   g.W = W.w_qkv; g.X = c.xn; g.X_lo = c.xn_lo; g.N = c.qkvN; g.K = c.d; g.out_f32 = c.qkv;
-  {
+  float* pool = l == 0 ? kv.pool_sum : nullptr;
+  if (c.use_tc) {
+    // bias, RoPE, q, cache append and pool update in the GEMM epilogue
+    g.qkv_bias = W.b_qkv; g.kv_len = kv.len; g.kv_seq_off = kv.seq_off; g.kv_cap = kv.cap;
+    g.kc = kv.k_cache[l]; g.vc = kv.v_cache[l]; g.q_out = c.q; g.pool = pool;
     ProfScope p(c, s, BUDDY_PROF_GEMM_QKV, 1, prof);
-    run_gemm(c, EPI_STORE_F32, g, l, 0, s);
-  }
-  {
+    run_gemm(c, EPI_QKV, g, l, 0, s);
+  } else {
+    {
+      ProfScope p(c, s, BUDDY_PROF_GEMM_QKV, 1, prof);
+      run_gemm(c, EPI_STORE_F32, g, l, 0, s);
+    }
     ProfScope p(c, s, BUDDY_PROF_QKV_FINALIZE, 1, prof);
-    launch_qkv_finalize(c, c.qkv, W.b_qkv, sel, kv, l, c.q, l == 0 ? kv.pool_sum : nullptr, s);
+    launch_qkv_finalize(c, c.qkv, W.b_qkv, sel, kv, l, c.q, pool, s);
   }
   {
     ProfScope p(c, s, BUDDY_PROF_ATTENTION, 2, prof);

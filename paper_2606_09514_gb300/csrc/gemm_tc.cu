@@ -49,6 +49,19 @@ struct TcParams {
   float* ws;
   int32_t* ctr;
   int32_t* status;
+  // EPI_QKV: bias, rotate-half RoPE at position len[seq], q out (fp32), K/V
+  // appended to the layer's cache, pooled first-layer V
+  const float* bias;
+  const float* rope_cos;
+  const float* rope_sin;
+  const int32_t* len;
+  const int64_t* seq_off;
+  const int32_t* cap;
+  bf16* kc;
+  bf16* vc;
+  float* q_out;
+  float* pool;
+  int nq, nkv, hd;
 };
 
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
@@ -66,7 +79,48 @@ __device__ __forceinline__ bool epi_bar_any(bool v) {
 template <int EPI, bool SPLIT>
 __device__ __forceinline__ void apply_epilogue(const TcParams& p, int tile, int row, int c0, int m,
                                                const float* v, float* xch) {
-  if (EPI == EPI_SWIGLU) {
+  if (EPI == EPI_QKV) {
+    // a 128-row tile holds whole heads (hd = 64 or 128): RoPE partners are
+    // rows of the same tile, exchanged through shared memory
+#pragma unroll
+    for (int i = 0; i < 16; ++i) xch[row * 17 + i] = v[i];
+    epi_bar();
+    const int nf = tile * 128 + row;
+    if (nf < p.N) {
+      const int hd = p.hd, half = hd >> 1;
+      const int head = nf / hd, e = nf - head * hd;
+      const bool lowh = e < half;
+      const int pr = lowh ? row + half : row - half;
+      const int ep = lowh ? e : e - half;
+      const float b0 = p.bias ? p.bias[nf] : 0.f;
+      const float bp = p.bias ? p.bias[lowh ? nf + half : nf - half] : 0.f;
+      const int kvd = p.nkv * hd;
+      for (int i = 0; i < 16; ++i) {
+        const int j = c0 + i;
+        if (j >= m) break;
+        const int seq = p.rows ? p.rows[j] : j;
+        const int pos = p.len[seq];
+        const float x = v[i] + b0;
+        if (head < p.nq + p.nkv) {
+          const float xp = xch[pr * 17 + i] + bp;
+          const float co = p.rope_cos[(size_t)pos * half + ep], si = p.rope_sin[(size_t)pos * half + ep];
+          const float y = lowh ? x * co - xp * si : x * co + xp * si;
+          if (head < p.nq) {
+            p.q_out[(size_t)j * p.nq * hd + nf] = y;
+          } else {
+            const int g = head - p.nq;
+            p.kc[kv_offset(p.seq_off, p.cap, seq, p.nkv, hd, g, pos) + e] = from_f<bf16>(y);
+          }
+        } else {
+          const int g = head - p.nq - p.nkv;
+          const bf16 vs = from_f<bf16>(x);
+          p.vc[kv_offset(p.seq_off, p.cap, seq, p.nkv, hd, g, pos) + e] = vs;
+          if (p.pool) p.pool[(size_t)seq * kvd + g * hd + e] += to_f(vs);
+        }
+      }
+    }
+    epi_bar();
+  } else if (EPI == EPI_SWIGLU) {
     // rows 0..63: gate of feature f = tile*64 + row; rows 64..127: up of the same f
     const bool up = row >= 64;
     const int r = row & 63;
@@ -123,7 +177,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __shared__ volatile int abort_flag;
   __shared__ volatile int consumed;
   __shared__ int last_flag;
-  __shared__ float xch[64 * 17];
+  __shared__ float xch[128 * 17];
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -322,13 +376,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (int c0 = 0; c0 < BN; c0 += 16) {
           ptx::tmem_ld16(taddr + c0, v);
 #pragma unroll
-          for (int i = 0; i < 16; ++i) __stcg(slot + (size_t)(c0 + i) * 128 + row, v[i]);
+          for (int i = 0; i < 16; ++i)
+            if (c0 + i < m) __stcg(slot + (size_t)(c0 + i) * 128 + row, v[i]);
         }
         ptx::tc_fence_before();
         if (lane == 0) ptx::mbar_arrive(&tempty_bar[acc]);
-        __threadfence();
         epi_bar();
         if (threadIdx.x == 64) {
+          __threadfence();
           const int old = atomicAdd(&p.ctr[tile], 1);
           last_flag = (old == p.splits - 1);
           if (last_flag) p.ctr[tile] = 0;
@@ -338,12 +393,23 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (last_flag) {
           __threadfence();
           for (int c0 = 0; c0 < BN; c0 += 16) {
+            const int nc = min(16, m - c0);
 #pragma unroll
             for (int i = 0; i < 16; ++i) v[i] = 0.f;
-            for (int s = 0; s < p.splits; ++s) {
-              const float* sl = p.ws + (size_t)(s * p.n_tiles + tile) * p.bn_max * 128;
+            // four splits' loads in flight per round, summed in split order
+            for (int s = 0; s < p.splits; s += 4) {
+              float t[4][16];
 #pragma unroll
-              for (int i = 0; i < 16; ++i) v[i] += __ldcg(sl + (size_t)(c0 + i) * 128 + row);
+              for (int q = 0; q < 4; ++q) {
+                const float* sl = p.ws + (size_t)((s + q) * p.n_tiles + tile) * p.bn_max * 128 + row;
+#pragma unroll
+                for (int i = 0; i < 16; ++i)
+                  t[q][i] = (s + q < p.splits && i < nc) ? __ldcg(sl + (size_t)(c0 + i) * 128) : 0.f;
+              }
+#pragma unroll
+              for (int q = 0; q < 4; ++q)
+#pragma unroll
+                for (int i = 0; i < 16; ++i) v[i] += t[q][i];
             }
             apply_epilogue<EPI, SPLIT>(p, tile, row, c0, m, v, xch);
           }
@@ -438,7 +504,7 @@ int gemm_tc_prepare(Ctx& c) {
   c.use_tc = gemm_tc_supported(c);
   if (!c.use_tc) return BUDDY_OK;
   c.tc_bn_max = std::max(16, (c.maxB + 15) & ~15);
-  const int smem_limit = 227 * 1024 - 8 * 1024;   // leave room for static shared memory
+  const int smem_limit = 227 * 1024 - 12 * 1024;  // leave room for static shared memory (~9.5 KiB)
   for (int v = 0; v < 2; ++v) {
     const uint32_t stage_bytes = kTileABytes + (uint32_t)(v + 1) * (uint32_t)c.tc_bn_max * 128u;
     c.tc_stages[v] = std::min(kTcMaxStages, (int)((smem_limit - 1024) / stage_bytes));
@@ -492,7 +558,9 @@ int gemm_tc_prepare(Ctx& c) {
       cudaFuncSetAttribute(gemm_tc_kernel<EPI_SWIGLU, false>, A, c.tc_smem[0]) ||
       cudaFuncSetAttribute(gemm_tc_kernel<EPI_STORE_F32, true>, A, c.tc_smem[1]) ||
       cudaFuncSetAttribute(gemm_tc_kernel<EPI_RESID, true>, A, c.tc_smem[1]) ||
-      cudaFuncSetAttribute(gemm_tc_kernel<EPI_SWIGLU, true>, A, c.tc_smem[1]))
+      cudaFuncSetAttribute(gemm_tc_kernel<EPI_SWIGLU, true>, A, c.tc_smem[1]) ||
+      cudaFuncSetAttribute(gemm_tc_kernel<EPI_QKV, false>, A, c.tc_smem[0]) ||
+      cudaFuncSetAttribute(gemm_tc_kernel<EPI_QKV, true>, A, c.tc_smem[1]))
     return BUDDY_ERR_CUDA;
   return BUDDY_OK;
 }
@@ -525,6 +593,19 @@ void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s) {
   p.ws = c.gemm_ws;
   p.ctr = c.gemm_ctr;
   p.status = c.status;
+  p.bias = a.qkv_bias;
+  p.rope_cos = c.rope_cos;
+  p.rope_sin = c.rope_sin;
+  p.len = a.kv_len;
+  p.seq_off = a.kv_seq_off;
+  p.cap = a.kv_cap;
+  p.kc = (bf16*)a.kc;
+  p.vc = (bf16*)a.vc;
+  p.q_out = a.q_out;
+  p.pool = a.pool;
+  p.nq = c.nq;
+  p.nkv = c.nkv;
+  p.hd = c.hd;
   const CUtensorMap& tw = c.tmaps_host[(size_t)a.layer * 4 + which];
   const int xi = which == 0 || which == 2 ? 0 : (which == 1 ? 1 : 2);
   const CUtensorMap& tx = c.tmaps_host[(size_t)c.L * 4 + xi];
@@ -533,6 +614,9 @@ void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s) {
   const size_t smem = c.tc_smem[v];
   if (a.split) {
     switch (epi) {
+      case EPI_QKV:
+        launch_k(gemm_tc_kernel<EPI_QKV, true>, grid, kTcThreads, smem, s, c.pdl, tw, tx, txlo, p);
+        break;
       case EPI_STORE_F32:
         launch_k(gemm_tc_kernel<EPI_STORE_F32, true>, grid, kTcThreads, smem, s, c.pdl, tw, tx, txlo, p);
         break;
@@ -544,6 +628,9 @@ void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s) {
     }
   } else {
     switch (epi) {
+      case EPI_QKV:
+        launch_k(gemm_tc_kernel<EPI_QKV, false>, grid, kTcThreads, smem, s, c.pdl, tw, tx, txlo, p);
+        break;
       case EPI_STORE_F32:
         launch_k(gemm_tc_kernel<EPI_STORE_F32, false>, grid, kTcThreads, smem, s, c.pdl, tw, tx, txlo, p);
         break;

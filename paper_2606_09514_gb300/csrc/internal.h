@@ -30,7 +30,7 @@ struct RowSel {
   int n;                  // count when `count` is null; upper bound otherwise
 };
 
-enum GemmEpi { EPI_STORE_F32 = 0, EPI_RESID = 1, EPI_SWIGLU = 2 };
+enum GemmEpi { EPI_STORE_F32 = 0, EPI_RESID = 1, EPI_SWIGLU = 2, EPI_QKV = 3 };
 
 struct GemmArgs {
   const void* W;          // [N_rows, K] (weight dtype)
@@ -47,6 +47,15 @@ struct GemmArgs {
   bool split;
   const float* resid_src; // EPI_RESID: dst[i] = src[i] + acc  (may equal dst)
   float* resid_dst;
+  // EPI_QKV (tensor-core path): QKV finalisation fused into the epilogue
+  const float* qkv_bias;
+  const int32_t* kv_len;
+  const int64_t* kv_seq_off;
+  const int32_t* kv_cap;
+  void* kc;
+  void* vc;
+  float* q_out;
+  float* pool;
   const int32_t* status;
   int layer;              // tensor-core path: which layer's weight map
   int which;              // 0 qkv, 1 o, 2 gate_up, 3 down

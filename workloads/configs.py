@@ -184,7 +184,17 @@ T_F32 = Workload("t-small-f32", SMALL_F32, batch=6, steps=2, seed=3,
                  ctx_kind="list", ctx_args=(0, 7, 64, 129, 31, 300),
                  k_kind="list", k_args=(1, 2, 3, 3, 2, 1))
 
-BY_NAME = {w.name: w for w in FULL_WORKLOADS + [T_GQA, T_QWEN, T_F32]}
+# Three-layer models with the benchmark shapes' per-layer sizes, for kernel
+# profiling captures that must stay small on the device.
+P_LLAMA3_3L_B1 = Workload("llama3-8b-3layer-b1", dataclasses.replace(LLAMA3_8B, name="llama3-8b-3layer", n_layers=3),
+                          batch=1, steps=16, seed=0, ctx_kind="fixed", ctx_args=(2048,),
+                          k_kind="fixed", k_args=(1,))
+P_QWEN_3L_B256 = Workload("qwen2.5-7b-3layer-b256",
+                          dataclasses.replace(QWEN25_7B, name="qwen2.5-7b-3layer", n_layers=3),
+                          batch=256, steps=8, seed=0, ctx_kind="lognormal", ctx_args=(2048, 0.5, 512, 8192),
+                          k_kind="fixed", k_args=(1,))
+
+BY_NAME = {w.name: w for w in FULL_WORKLOADS + [T_GQA, T_QWEN, T_F32, P_LLAMA3_3L_B1, P_QWEN_3L_B256]}
 
 
 def scaled(w: Workload, *, batch: Optional[int] = None, steps: Optional[int] = None,
