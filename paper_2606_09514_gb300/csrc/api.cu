@@ -402,6 +402,16 @@ static int enqueue_step(buddy_ctx* x, const buddy_kv_state& kv, const StepIO& io
     CK(cudaMemcpyAsync(hcount, c.count, sizeof(int32_t) * c.L, cudaMemcpyDeviceToHost, s));
     CK(cudaStreamSynchronize(s));
   }
+  cudaGraphConditionalHandle handles[kMaxLayers];
+  if (capture) {
+    // one handle per middle layer, all set by a single kernel after compaction
+    cudaGraph_t g = nullptr;
+    cudaStreamCaptureStatus st;
+    CK(cudaStreamGetCaptureInfo(s, &st, nullptr, &g, nullptr, nullptr, nullptr));
+    for (int l = 1; l < c.L - 1; ++l)
+      CK(cudaGraphConditionalHandleCreate(&handles[l - 1], g, 0, cudaGraphCondAssignDefault));
+    launch_set_conditionals(handles, c.L - 2, c.count, c.status, s);
+  }
   for (int l = 1; l < c.L - 1; ++l) {
     const RowSel sel{c.rows + (size_t)l * B, c.count + l, B};
     if (!capture) {
@@ -410,17 +420,13 @@ static int enqueue_step(buddy_ctx* x, const buddy_kv_state& kv, const StepIO& io
     }
     cudaGraph_t g = nullptr;
     cudaStreamCaptureStatus st;
-    CK(cudaStreamGetCaptureInfo(s, &st, nullptr, &g, nullptr, nullptr, nullptr));
-    cudaGraphConditionalHandle h;
-    CK(cudaGraphConditionalHandleCreate(&h, g, 0, cudaGraphCondAssignDefault));
-    launch_set_conditional(h, c.count + l, c.status, s);
     const cudaGraphNode_t* deps = nullptr;
     const cudaGraphEdgeData* edata = nullptr;
     size_t ndeps = 0;
     CK(cudaStreamGetCaptureInfo(s, &st, nullptr, &g, &deps, &edata, &ndeps));
     cudaGraphNodeParams p{};
     p.type = cudaGraphNodeTypeConditional;
-    p.conditional.handle = h;
+    p.conditional.handle = handles[l - 1];
     p.conditional.type = cudaGraphCondTypeIf;
     p.conditional.size = 1;
     cudaGraphNode_t node;
@@ -464,6 +470,11 @@ static int run_step(buddy_ctx* x, const buddy_kv_state* kv, const StepIO& io, cu
   key.kvp.push_back(kv->pool_sum);
   auto it = c.graphs.find(key);
   if (it == c.graphs.end()) {
+    if (c.graphs.size() >= 16) {   // bounded cache: drop an arbitrary old entry
+      CK(cudaStreamSynchronize(s));
+      cudaGraphExecDestroy(c.graphs.begin()->second);
+      c.graphs.erase(c.graphs.begin());
+    }
     cudaStream_t cs = x->cap_stream;
     CK(cudaStreamBeginCapture(cs, cudaStreamCaptureModeRelaxed));
     int rc = enqueue_step(x, *kv, io, cs, true);

@@ -471,8 +471,9 @@ static void gemm_shape(const Ctx& c, int which, int* N, int* K, int* tiles) {
   }
 }
 
-// Split-K factor: every split gets >= 4 K-blocks; maximise the fraction of the
-// last wave of persistent CTAs that is busy, prefer fewer splits on ties.
+// Split-K factor: the smallest one whose last wave of persistent CTAs is at
+// least 80% busy (every split >= 4 K-blocks); fewer splits mean fewer
+// per-unit epilogues and partial sums.  Falls back to the best efficiency.
 static int choose_splits(int tiles, int kb, int sms) {
   int best = 1;
   double best_eff = -1.0;
@@ -482,6 +483,7 @@ static int choose_splits(int tiles, int kb, int sms) {
     const int units = tiles * s;
     const int waves = (units + sms - 1) / sms;
     const double eff = (double)units / (double)(waves * sms);
+    if (eff >= 0.8) return s;
     if (eff > best_eff + 0.02) {
       best_eff = eff;
       best = s;
