@@ -223,7 +223,9 @@ BUDDY_API int buddy_set_options(buddy_ctx* ctx, int32_t use_graph);
 enum {
   BUDDY_PROF_CHECK = 0, BUDDY_PROF_RMSNORM, BUDDY_PROF_GEMM_QKV, BUDDY_PROF_QKV_FINALIZE,
   BUDDY_PROF_ATTENTION, BUDDY_PROF_GEMM_O, BUDDY_PROF_GEMM_GATE_UP, BUDDY_PROF_GEMM_DOWN,
-  BUDDY_PROF_ROUTE, BUDDY_PROF_COMPACT, BUDDY_PROF_OTHER, BUDDY_PROF_NCLASS
+  BUDDY_PROF_ROUTE, BUDDY_PROF_COMPACT, BUDDY_PROF_OTHER,
+  BUDDY_PROF_LAYER,   /* a whole block as one persistent kernel (small batches) */
+  BUDDY_PROF_NCLASS
 };
 
 /* Per-kernel-class timing.  With on != 0, direct-launch decode steps

@@ -147,4 +147,14 @@ __device__ __forceinline__ void apply_epilogue(const TcParams& p, int tile, int 
   }
 }
 
+// GEMM shapes: which = 0 qkv, 1 o, 2 gate_up, 3 down
+inline void gemm_shape(const Ctx& c, int which, int* N, int* K, int* tiles) {
+  switch (which) {
+    case 0: *N = c.qkvN; *K = c.d; *tiles = (c.qkvN + 127) / 128; break;
+    case 1: *N = c.d; *K = c.qd; *tiles = (c.d + 127) / 128; break;
+    case 2: *N = c.F; *K = c.d; *tiles = (c.F + 63) / 64; break;
+    default: *N = c.d; *K = c.F; *tiles = (c.d + 127) / 128; break;
+  }
+}
+
 }  // namespace buddy

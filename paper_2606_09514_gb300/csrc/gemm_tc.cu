@@ -326,16 +326,6 @@ static bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t K
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// GEMM shapes: which = 0 qkv, 1 o, 2 gate_up, 3 down
-static void gemm_shape(const Ctx& c, int which, int* N, int* K, int* tiles) {
-  switch (which) {
-    case 0: *N = c.qkvN; *K = c.d; *tiles = (c.qkvN + 127) / 128; break;
-    case 1: *N = c.d; *K = c.qd; *tiles = (c.d + 127) / 128; break;
-    case 2: *N = c.F; *K = c.d; *tiles = (c.F + 63) / 64; break;
-    default: *N = c.d; *K = c.F; *tiles = (c.d + 127) / 128; break;
-  }
-}
-
 // Split-K factor: the smallest one whose last wave of persistent CTAs is at
 // least 80% busy (every split >= 4 K-blocks); fewer splits mean fewer
 // per-unit epilogues and partial sums.  Falls back to the best efficiency.
@@ -369,6 +359,7 @@ bool gemm_tc_supported(const Ctx& c) {
 
 int gemm_tc_prepare(Ctx& c) {
   c.use_tc = gemm_tc_supported(c);
+  c.use_lk = false;
   if (!c.use_tc) return BUDDY_OK;
   c.tc_bn_max = std::max(16, (c.maxB + 15) & ~15);
   const int smem_limit = 227 * 1024 - 12 * 1024;  // leave room for static shared memory (~9.5 KiB)
@@ -419,6 +410,12 @@ int gemm_tc_prepare(Ctx& c) {
     c.gemm_ctr_n = max_tiles;
   }
   if (cudaMemset(c.gemm_ctr, 0, c.gemm_ctr_n * sizeof(int32_t)) != cudaSuccess) return BUDDY_ERR_CUDA;
+  const char* lk_env = getenv("BUDDY_LAYER_KERNEL");
+  c.use_lk = layer_kernel_supported(c) && lk_env && lk_env[0] == '1';   // opt-in
+  if (c.use_lk && !c.lk_bar) {
+    if (cudaMalloc(&c.lk_bar, 2 * sizeof(unsigned)) != cudaSuccess) return BUDDY_ERR_CUDA;
+    if (cudaMemset(c.lk_bar, 0, 2 * sizeof(unsigned)) != cudaSuccess) return BUDDY_ERR_CUDA;
+  }
   const cudaFuncAttribute A = cudaFuncAttributeMaxDynamicSharedMemorySize;
   if (cudaFuncSetAttribute(gemm_tc_kernel<EPI_STORE_F32, false>, A, c.tc_smem[0]) ||
       cudaFuncSetAttribute(gemm_tc_kernel<EPI_RESID, false>, A, c.tc_smem[0]) ||

@@ -113,6 +113,10 @@ void launch_set_conditionals(const cudaGraphConditionalHandle* h, int n, const i
 // GEMMs (gemm_simt.cu, gemm_tc.cu)
 void launch_gemm_simt(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s);
 bool gemm_tc_supported(const Ctx& c);
+// layer_kernel.cu: one executed block as one persistent cooperative kernel
+bool layer_kernel_supported(const Ctx& c);
+bool launch_layer_kernel(const Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, const float* src, float* H,
+                         cudaStream_t s);
 void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s);
 
 struct Ctx {
@@ -164,6 +168,8 @@ struct Ctx {
   int tc_bn_max = 16, tc_stages[2] = {1, 1}, tc_smem[2] = {0, 0};   // [plain, split activations]
   uint32_t tc_stage_bytes[2] = {0, 0}, tc_tmem_cols = 32;
   int tc_splits[4] = {1, 1, 1, 1}, tc_tiles[4] = {1, 1, 1, 1};
+  bool use_lk = false;                    // per-layer persistent kernel (small batches)
+  unsigned* lk_bar = nullptr;             // its grid barrier [arrivals, generation]
   float* gemm_ws = nullptr;
   size_t gemm_ws_elems = 0;
   int32_t* gemm_ctr = nullptr;
