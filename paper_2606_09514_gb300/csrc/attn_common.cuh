@@ -136,7 +136,7 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
   constexpr int V16 = HD * (int)sizeof(T) / 16;  // 16-byte pieces per row
   constexpr int E16 = 16 / sizeof(T);            // elements per piece
   const int G = nq / nkv;
-    T* Kb0 = reinterpret_cast<T*>(smem);                          // 2 x [kChunk][KROW]
+  T* Kb0 = reinterpret_cast<T*>(smem);                          // 2 x [kChunk][KROW]
   T* Vb0 = Kb0 + 2 * kChunk * KROW;                              // 2 x [kChunk][HD]
   float* qs = reinterpret_cast<float*>(Vb0 + 2 * kChunk * HD);   // [G][HD]
   float* ps = qs + G * HD;                                       // [G][kChunk]
@@ -353,20 +353,35 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
           if (lane == 0) lrun_s[h] = lsum;
         }
         sync();
-        for (int x = tid; x < G * HD; x += kAttnThreads) {
-          const int h = x / HD, ee = x - h * HD;
+        // four consecutive channels per thread; the partials of eight spans
+        // are loaded together, then accumulated in span order
+        for (int x4 = tid; x4 < G * HD / 4; x4 += kAttnThreads) {
+          const int h = (x4 * 4) / HD, ee = x4 * 4 - h * HD;
           const float* pa0 = part_acc + ((size_t)j * nq + g * G + h) * max_spans * HD + ee;
           const float* wh = wch + h * max_spans;
-          float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-          int cc = 0;
-          for (; cc + 4 <= nsp; cc += 4) {
-            a0 += __ldcg(pa0 + (size_t)(cc + 0) * HD) * wh[cc + 0];
-            a1 += __ldcg(pa0 + (size_t)(cc + 1) * HD) * wh[cc + 1];
-            a2 += __ldcg(pa0 + (size_t)(cc + 2) * HD) * wh[cc + 2];
-            a3 += __ldcg(pa0 + (size_t)(cc + 3) * HD) * wh[cc + 3];
+          float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+          for (int c0 = 0; c0 < nsp; c0 += 8) {
+            float4 t[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+              if (c0 + k < nsp) t[k] = __ldcg(reinterpret_cast<const float4*>(pa0 + (size_t)(c0 + k) * HD));
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              if (c0 + k < nsp) {
+                const float w = wh[c0 + k];
+                a.x += t[k].x * w;
+                a.y += t[k].y * w;
+                a.z += t[k].z * w;
+                a.w += t[k].w * w;
+              }
+            }
           }
-          for (; cc < nsp; ++cc) a0 += __ldcg(pa0 + (size_t)cc * HD) * wh[cc];
-          store_out(out, out_lo, obase + (size_t)h * HD + ee, ((a0 + a1) + (a2 + a3)) / lrun_s[h]);
+          const float l = lrun_s[h];
+          const size_t o = obase + (size_t)h * HD + ee;
+          store_out(out, out_lo, o + 0, a.x / l);
+          store_out(out, out_lo, o + 1, a.y / l);
+          store_out(out, out_lo, o + 2, a.z / l);
+          store_out(out, out_lo, o + 3, a.w / l);
         }
       }
     }

@@ -1,6 +1,30 @@
-// Shared pieces of the tensor-core GEMM (gemm_tc.cu) and the per-layer
-// persistent kernel (layer_kernel.cu): tile constants, parameters of one GEMM,
-// and the epilogues applied to a 128-feature x 16-row block of results.
+// Building blocks of the tensor-core decode GEMM, shared by the GEMM kernel
+// (gemm_tc.cu) and the per-layer persistent kernel (layer_kernel.cu).
+//
+//   C[j][n] = sum_k X[j][k] * W[n][k]      (j < m active rows, n < N features)
+//
+// Orientation.  A tcgen05.mma instruction (K = 16) takes about 150 cycles
+// whatever its M and N, so a decode GEMM, bound by streaming W, must move as
+// many weight bytes per instruction as it can.  The active rows are therefore
+// the MMA's M side (one or two 128-row M-tiles; rows past m are never read
+// back) and a tile of bw = 256 weight rows is its N side: 8 KiB of weights per
+// instruction.  (With the weights as M and the rows as N, an instruction moves
+// 4 KiB and the instruction rate caps an SM's weight stream near 5 TB/s for
+// the whole GPU.)
+//
+// A stage of the shared-memory ring holds, for one 64-column K block, the
+// activation region of each M-tile (then, for the first layer, the regions of
+// the bf16 remainder terms) followed by the weight tile [bw rows][128 B], all
+// in the 128-byte-swizzled K-major layout.  Only round16(m) activation rows are
+// loaded; an M-tile operand always spans 128 rows, so its unused rows read the
+// bytes that follow within the stage (their results are discarded).
+//
+// The accumulator of a unit (tile, K split) is mt x 256 fp32 TMEM columns.
+// Small batches use a short ring (about 100 KiB) and one accumulator, so that
+// two GEMM CTAs fit on an SM: under programmatic dependent launch the next
+// GEMM's CTAs start streaming their weights while the current one finishes.
+// Otherwise the ring fills shared memory and, with one M-tile, two
+// accumulators let the MMAs of the next unit overlap the epilogue.
 #pragma once
 
 #include <cuda.h>
@@ -13,15 +37,19 @@ namespace buddy {
 
 constexpr int kTcThreads = 192;
 constexpr int kTcMaxStages = 16;
-constexpr int kTileK = 64;
-constexpr uint32_t kTileABytes = 128 * kTileK * 2;   // 16 KiB weight tile
-constexpr uint64_t kWaitLimitNs = 4000000000ull;     // 4 s
+constexpr int kTileK = 64;                       // K columns per stage (128 B of bf16)
+constexpr uint32_t kXTileMax = 128 * 128;        // bytes one M-tile operand spans
+constexpr int kTileN = 256;                      // weight rows per tile (MMA N)
+constexpr uint64_t kWaitLimitNs = 4000000000ull; // 4 s
 
 struct TcParams {
   int N, K;
   int n_tiles, splits, kb_total, kb_per_split, units;
-  int bn_max, stages;
-  uint32_t stage_bytes, tmem_cols;
+  int bw, mt;              // weight rows per tile, M-tiles
+  uint32_t w_off;          // byte offset of the weight tile in a stage
+  int rows_max;            // rows of a workspace slot (round16 of the batch bound)
+  int stages, acc_bufs;
+  uint32_t stage_bytes, xr, tmem_cols;   // xr: bytes of one M-tile's activation region
   const int32_t* rows;
   const int32_t* count;
   int n;
@@ -60,100 +88,267 @@ __device__ __forceinline__ bool epi_bar_any(bool v) {
   return r != 0;
 }
 
-template <int EPI, bool SPLIT>
-__device__ __forceinline__ void apply_epilogue(const TcParams& p, int tile, int row, int c0, int m,
-                                               const float* v, float* xch) {
-  if (EPI == EPI_QKV) {
-    // a 128-row tile holds whole heads (hd = 64 or 128): RoPE partners are
-    // rows of the same tile, exchanged through shared memory
-#pragma unroll
-    for (int i = 0; i < 16; ++i) xch[row * 17 + i] = v[i];
-    epi_bar();
-    const int nf = tile * 128 + row;
-    if (nf < p.N) {
-      const int hd = p.hd, half = hd >> 1;
-      const int head = nf / hd, e = nf - head * hd;
-      const bool lowh = e < half;
-      const int pr = lowh ? row + half : row - half;
-      const int ep = lowh ? e : e - half;
-      const float b0 = p.bias ? p.bias[nf] : 0.f;
-      const float bp = p.bias ? p.bias[lowh ? nf + half : nf - half] : 0.f;
-      const int kvd = p.nkv * hd;
-      for (int i = 0; i < 16; ++i) {
-        const int j = c0 + i;
-        if (j >= m) break;
-        const int seq = p.rows ? p.rows[j] : j;
-        const int pos = p.len[seq];
-        const float x = v[i] + b0;
-        if (head < p.nq + p.nkv) {
-          const float xp = xch[pr * 17 + i] + bp;
-          const float co = p.rope_cos[(size_t)pos * half + ep], si = p.rope_sin[(size_t)pos * half + ep];
-          const float y = lowh ? x * co - xp * si : x * co + xp * si;
-          if (head < p.nq) {
-            p.q_out[(size_t)j * p.nq * hd + nf] = y;
-          } else {
-            const int g = head - p.nq;
-            p.kc[kv_offset(p.seq_off, p.cap, seq, p.nkv, hd, g, pos) + e] = from_f<bf16>(y);
-          }
-        } else {
-          const int g = head - p.nq - p.nkv;
-          const bf16 vs = from_f<bf16>(x);
-          p.vc[kv_offset(p.seq_off, p.cap, seq, p.nkv, hd, g, pos) + e] = vs;
-          if (p.pool) p.pool[(size_t)seq * kvd + g * hd + e] += to_f(vs);
-        }
-      }
-    }
-    epi_bar();
-  } else if (EPI == EPI_SWIGLU) {
-    // rows 0..63: gate of feature f = tile*64 + row; rows 64..127: up of the same f
-    const bool up = row >= 64;
-    const int r = row & 63;
-    if (up) {
-#pragma unroll
-      for (int i = 0; i < 16; ++i) xch[r * 17 + i] = v[i];
-    }
-    epi_bar();
-    if (!up) {
-      const int f = tile * 64 + r;
-      if (f < p.N) {
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const int j = c0 + i;
-          if (j < m) {
-            const float a = silu_f(v[i]) * xch[r * 17 + i];
-            const bf16 hi = from_f<bf16>(a);
-            p.out_act[(size_t)j * p.N + f] = hi;
-            if (SPLIT) p.out_act_lo[(size_t)j * p.N + f] = from_f<bf16>(a - to_f(hi));
-          }
-        }
-      }
-    }
-    epi_bar();
+__device__ __forceinline__ int round16(int x) { return (x + 15) & ~15; }
+
+// ---------------------------------------------------------------------------
+// Loads of one stage.  The caller has set the barrier's expected bytes.
+// ---------------------------------------------------------------------------
+// Weight tile `tile` at K block kb.  SwiGLU: the first bw/2 rows are gate rows
+// f0.., the next bw/2 the matching up rows N + f0.. (N = F).
+template <int EPI>
+__device__ __forceinline__ void tc_load_w(uint8_t* stage, const CUtensorMap* tw, uint64_t* bar, const TcParams& p,
+                                          int tile, int kb, uint64_t pol) {
+  uint8_t* st = stage + p.w_off;
+  if (EPI == EPI_SWIGLU) {
+    const int h = p.bw >> 1;
+    ptx::tma_load_2d_hint(st, tw, bar, kb * kTileK, tile * h, pol);
+    ptx::tma_load_2d_hint(st + h * 128, tw, bar, kb * kTileK, p.N + tile * h, pol);
   } else {
-    const int nf = tile * 128 + row;
-    if (nf >= p.N) return;
+    ptx::tma_load_2d_hint(st, tw, bar, kb * kTileK, tile * p.bw, pol);
+  }
+}
+
+__device__ __forceinline__ uint32_t tc_x_bytes(int m, bool split) {
+  return (split ? 2u : 1u) * (uint32_t)round16(m) * 128u;
+}
+
+// Activation rows 0..round16(m)-1 at K block kb, 16 rows per copy.
+template <bool SPLIT>
+__device__ __forceinline__ void tc_load_x(uint8_t* st, const CUtensorMap* tx, const CUtensorMap* txlo, uint64_t* bar,
+                                          const TcParams& p, int m, int kb) {
+  uint8_t* x0 = st;
+  uint8_t* l0 = x0 + p.mt * p.xr;
+  for (int r0 = 0; r0 < m; r0 += 16) {
+    const uint32_t off = (uint32_t)(r0 >> 7) * p.xr + (uint32_t)(r0 & 127) * 128u;
+    ptx::tma_load_2d(x0 + off, tx, bar, kb * kTileK, r0);
+    if (SPLIT) ptx::tma_load_2d(l0 + off, txlo, bar, kb * kTileK, r0);
+  }
+}
+
+// MMAs of one stage into accumulator column `d`: every M-tile holding rows
+// (and, SPLIT, its remainder terms into the same accumulator).
+template <bool SPLIT>
+__device__ __forceinline__ void tc_mma_stage(const uint8_t* st, uint32_t d, const TcParams& p, int m,
+                                             uint32_t idesc, bool first) {
+  const uint64_t dw = ptx::smem_desc_sw128(st + p.w_off);
+  for (int t = 0; t < p.mt && t * 128 < m; ++t) {
+    const uint8_t* xt = st + t * p.xr;
+    const uint64_t dx = ptx::smem_desc_sw128(xt);
+    const uint64_t dl = ptx::smem_desc_sw128(xt + p.mt * p.xr);
+    const uint32_t dt = d + (uint32_t)(t * p.bw);
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      const int j = c0 + i;
-      if (j >= m) break;
-      if (EPI == EPI_STORE_F32) {
-        p.out_f32[(size_t)j * p.N + nf] = v[i];
-      } else {
-        const int seq = p.rows ? p.rows[j] : j;
-        const size_t o = (size_t)seq * p.N + nf;
-        p.resid_dst[o] = p.resid_src[o] + v[i];
-      }
+    for (int k = 0; k < kTileK / 16; ++k) {
+      ptx::mma_bf16(dt, dx + 2ull * k, dw + 2ull * k, idesc, (!first || k > 0) ? 1u : 0u);
+      if (SPLIT) ptx::mma_bf16(dt, dl + 2ull * k, dw + 2ull * k, idesc, 1u);
     }
   }
 }
 
-// GEMM shapes: which = 0 qkv, 1 o, 2 gate_up, 3 down
+// ---------------------------------------------------------------------------
+// Epilogue of row j, accumulator columns c..c+3 of a tile (`v`), with the
+// partner columns `vp` where the epilogue pairs columns (SwiGLU: the up rows
+// bw/2 further on; QKV: the other half of each rotate-half pair, hd/2 further).
+// ---------------------------------------------------------------------------
+template <int EPI>
+__device__ __forceinline__ int tc_partner_off(const TcParams& p) {
+  return EPI == EPI_SWIGLU ? (p.bw >> 1) : (EPI == EPI_QKV ? (p.hd >> 1) : 0);
+}
+// Work items of one tile's epilogue: (row, group of 4 primary columns).
+template <int EPI>
+__device__ __forceinline__ int tc_groups(const TcParams& p) {
+  return EPI == EPI_SWIGLU || EPI == EPI_QKV ? p.bw / 8 : p.bw / 4;
+}
+template <int EPI>
+__device__ __forceinline__ int tc_group_col(const TcParams& p, int g) {
+  if (EPI == EPI_QKV) {
+    const int per = p.hd >> 3;   // groups in the low half of a head
+    return (g / per) * p.hd + (g % per) * 4;
+  }
+  return g * 4;
+}
+
+template <int EPI, bool SPLIT>
+__device__ __forceinline__ void tc_apply4(const TcParams& p, int tile, int j, int c, const float* v, const float* vp,
+                                          const float* rs) {
+  if (EPI == EPI_SWIGLU) {
+    const int f0 = tile * (p.bw >> 1) + c;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int f = f0 + i;
+      if (f < p.N) {
+        const float a = silu_f(v[i]) * vp[i];
+        const bf16 hi = from_f<bf16>(a);
+        p.out_act[(size_t)j * p.N + f] = hi;
+        if (SPLIT) p.out_act_lo[(size_t)j * p.N + f] = from_f<bf16>(a - to_f(hi));
+      }
+    }
+  } else if (EPI == EPI_QKV) {
+    const int hd = p.hd, half = hd >> 1;
+    const int n0 = tile * p.bw + c;
+    if (n0 >= p.N) return;   // heads are whole: a group and its partner are in or out together
+    const int head = n0 / hd, e0 = n0 - head * hd;
+    const int seq = p.rows ? p.rows[j] : j;
+    const int pos = p.len[seq];
+    float x[4], xp[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      x[i] = v[i] + (p.bias ? p.bias[n0 + i] : 0.f);
+      xp[i] = vp[i] + (p.bias ? p.bias[n0 + half + i] : 0.f);
+    }
+    if (head < p.nq + p.nkv) {
+      const float* co = p.rope_cos + (size_t)pos * half + e0;
+      const float* si = p.rope_sin + (size_t)pos * half + e0;
+      float lo[4], hi[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        lo[i] = x[i] * co[i] - xp[i] * si[i];
+        hi[i] = xp[i] * co[i] + x[i] * si[i];
+      }
+      if (head < p.nq) {
+        float* q = p.q_out + (size_t)j * p.nq * hd + n0;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          q[i] = lo[i];
+          q[half + i] = hi[i];
+        }
+      } else {
+        bf16* k = p.kc + kv_offset(p.seq_off, p.cap, seq, p.nkv, hd, head - p.nq, pos) + e0;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          k[i] = from_f<bf16>(lo[i]);
+          k[half + i] = from_f<bf16>(hi[i]);
+        }
+      }
+    } else {
+      const int g = head - p.nq - p.nkv;
+      bf16* vv = p.vc + kv_offset(p.seq_off, p.cap, seq, p.nkv, hd, g, pos) + e0;
+      float* pl = p.pool ? p.pool + (size_t)seq * p.nkv * hd + g * hd + e0 : nullptr;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const bf16 a = from_f<bf16>(x[i]), b = from_f<bf16>(xp[i]);
+        vv[i] = a;
+        vv[half + i] = b;
+        if (pl) {
+          pl[i] += to_f(a);
+          pl[half + i] += to_f(b);
+        }
+      }
+    }
+  } else {
+    const int n0 = tile * p.bw + c;
+    if (EPI == EPI_STORE_F32) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (n0 + i < p.N) p.out_f32[(size_t)j * p.N + n0 + i] = v[i];
+    } else {
+      const int seq = p.rows ? p.rows[j] : j;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (n0 + i < p.N) p.resid_dst[(size_t)seq * p.N + n0 + i] = rs[i] + v[i];
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Epilogue of one unit by the four epilogue warps (128 threads).  Warp w reads
+// TMEM lanes 32*(w%4).. (rows of each M-tile) and writes the unit's
+// accumulator rows j < m to its workspace slot; the accumulator is released
+// (tempty) right after.  The CTA that completes a tile (the last of its K
+// splits, or the only one) then applies the epilogue with all 128 threads over
+// (row, 4-column group) items, summing the splits' slots in split order
+// (deterministic).  Returns whether this CTA finished the tile.
+// ---------------------------------------------------------------------------
+template <int EPI, bool SPLIT>
+__device__ __forceinline__ void tc_epilogue_unit(const TcParams& p, int u, int m, uint32_t tacc, uint64_t* tempty,
+                                                 int* last_flag) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int q = warp & 3;   // TMEM lane quarter this warp may access
+  const int tile = u % p.n_tiles;
+  float* slot = p.ws + (size_t)u * p.rows_max * p.bw;
+  for (int t = 0; t < p.mt; ++t) {
+    if (t * 128 + q * 32 >= m) continue;   // warp-uniform
+    const int j = t * 128 + q * 32 + lane;
+    const uint32_t ta = tacc + ((uint32_t)(q * 32) << 16) + (uint32_t)(t * p.bw);
+    for (int c0 = 0; c0 < p.bw; c0 += 64) {
+      float v[64];
+      ptx::tmem_ld64(ta + c0, v);
+      if (j < m) {
+        float4* d = reinterpret_cast<float4*>(slot + (size_t)j * p.bw + c0);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) __stcg(d + i, make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]));
+      }
+    }
+  }
+  ptx::tc_fence_before();
+  if (lane == 0) ptx::mbar_arrive(tempty);
+  epi_bar();
+  const int et = threadIdx.x & 127;
+  if (et == 0) {
+    __threadfence();
+    int last = 1;
+    if (p.splits > 1) {
+      const int old = atomicAdd(&p.ctr[tile], 1);
+      last = old == p.splits - 1;
+      if (last) p.ctr[tile] = 0;
+    }
+    *last_flag = last;
+    __threadfence();
+  }
+  epi_bar();
+  if (*last_flag) {
+    __threadfence();
+    const int po = tc_partner_off<EPI>(p);
+    const int ng = tc_groups<EPI>(p);
+    const int items = m * ng;
+    const size_t sstride = (size_t)p.n_tiles * p.rows_max * p.bw;   // one split's slots
+    const float* base = p.ws + (size_t)tile * p.rows_max * p.bw;
+    // one item per thread per round; the partials of up to eight splits (and
+    // the residual) are loaded together, then summed in split order
+    for (int it = et; it < items; it += 128) {
+      const int j = it / ng, c = tc_group_col<EPI>(p, it - j * ng);
+      const float* sl = base + (size_t)j * p.bw + c;
+      float v[4] = {0.f, 0.f, 0.f, 0.f}, vp[4] = {0.f, 0.f, 0.f, 0.f}, rs[4] = {0.f, 0.f, 0.f, 0.f};
+      if (EPI == EPI_RESID) {
+        const int seq = p.rows ? p.rows[j] : j;
+        const int n0 = tile * p.bw + c;
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (n0 + i < p.N) rs[i] = p.resid_src[(size_t)seq * p.N + n0 + i];
+      }
+      for (int s0 = 0; s0 < p.splits; s0 += 8) {
+        float4 x[8], y[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          if (s0 + k < p.splits) {
+            x[k] = __ldcg(reinterpret_cast<const float4*>(sl + (size_t)(s0 + k) * sstride));
+            if (po) y[k] = __ldcg(reinterpret_cast<const float4*>(sl + (size_t)(s0 + k) * sstride + po));
+          }
+        }
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          if (s0 + k < p.splits) {
+            v[0] += x[k].x; v[1] += x[k].y; v[2] += x[k].z; v[3] += x[k].w;
+            if (po) {
+              vp[0] += y[k].x; vp[1] += y[k].y; vp[2] += y[k].z; vp[3] += y[k].w;
+            }
+          }
+        }
+      }
+      tc_apply4<EPI, SPLIT>(p, tile, j, c, v, vp, rs);
+    }
+  }
+  epi_bar();
+}
+
+// GEMM shapes: which = 0 qkv, 1 o, 2 gate_up, 3 down; tiles of bw features
+// (gate/up: bw/2 features, each with its gate and up rows)
 inline void gemm_shape(const Ctx& c, int which, int* N, int* K, int* tiles) {
+  const int bw = c.tc_bw;
   switch (which) {
-    case 0: *N = c.qkvN; *K = c.d; *tiles = (c.qkvN + 127) / 128; break;
-    case 1: *N = c.d; *K = c.qd; *tiles = (c.d + 127) / 128; break;
-    case 2: *N = c.F; *K = c.d; *tiles = (c.F + 63) / 64; break;
-    default: *N = c.d; *K = c.F; *tiles = (c.d + 127) / 128; break;
+    case 0: *N = c.qkvN; *K = c.d; *tiles = (c.qkvN + bw - 1) / bw; break;
+    case 1: *N = c.d; *K = c.qd; *tiles = (c.d + bw - 1) / bw; break;
+    case 2: *N = c.F; *K = c.d; *tiles = (c.F + bw / 2 - 1) / (bw / 2); break;
+    default: *N = c.d; *K = c.F; *tiles = (c.d + bw - 1) / bw; break;
   }
 }
 

@@ -2,18 +2,17 @@
 //
 //   C[j][n] = sum_k X[j][k] * W[n][k]      (j < m active rows, n < N features)
 //
-// Decode GEMMs are skinny (m = 1..256) and bound by streaming W from HBM, so
-// the operands are swapped: a 128-row weight tile is the MMA's M side and the
-// m active rows (padded to a multiple of 16) are its N side.  Both operands are
-// K-major bf16 tiles of 64 columns staged in shared memory by TMA with 128-byte
-// swizzle; tcgen05.mma accumulates fp32 in TMEM.  Persistent CTAs (one per SM)
-// walk work units (weight tile, K split); warp 0 issues TMA loads into a ring
-// of stages, warp 1 issues the MMAs, warps 2-5 drain TMEM (double-buffered
-// accumulators) and run the epilogue.  A tile split over K is finished by the
-// last CTA to arrive, which sums the partials in split order (deterministic).
+// Decode GEMMs are skinny (m = 1..256) and bound by streaming W from HBM.  The
+// tile geometry, the ring stage layout and the epilogues are described in
+// gemm_common.cuh.  Persistent CTAs (one per SM) walk work units (weight tile,
+// K split); warp 0 issues TMA loads into a ring of stages, warp 1 issues the
+// tcgen05 MMAs (accumulating fp32 in TMEM), warps 2-5 drain TMEM and run the
+// epilogue.  A tile split over K is finished by the last CTA to arrive, which
+// sums the partials in split order (deterministic).
 //
 // Epilogues: fp32 store; residual add into the (row-gathered) hidden state;
-// SwiGLU, where a tile holds 64 gate rows and the matching 64 up rows.
+// SwiGLU (a tile holds 128 gate rows and the matching 128 up rows); QKV
+// finalisation (bias, RoPE, q, K/V cache append, pooled first-layer V).
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -42,7 +41,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __shared__ volatile int abort_flag;
   __shared__ volatile int consumed;
   __shared__ int last_flag;
-  __shared__ float xch[128 * 17];
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -72,6 +70,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem_base = tmem_slot;
+  const uint32_t w_bytes = (uint32_t)p.bw * 128u;
 
   // Weight tiles depend on nothing an earlier kernel writes: start streaming
   // the first `stages` of them before waiting for the predecessor.
@@ -83,14 +82,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const int tile = u % p.n_tiles, split = u / p.n_tiles;
       const int kb0 = split * p.kb_per_split, kb1 = min(p.kb_total, kb0 + p.kb_per_split);
       for (int kb = kb0; kb < kb1 && npre < p.stages; ++kb, ++npre) {
-        uint8_t* a = smem + (size_t)npre * p.stage_bytes;
-        ptx::mbar_expect_tx(&full_bar[npre], kTileABytes);
-        if (EPI == EPI_SWIGLU) {
-          ptx::tma_load_2d_hint(a, &tw, &full_bar[npre], kb * kTileK, tile * 64, pol);
-          ptx::tma_load_2d_hint(a + kTileABytes / 2, &tw, &full_bar[npre], kb * kTileK, p.N + tile * 64, pol);
-        } else {
-          ptx::tma_load_2d_hint(a, &tw, &full_bar[npre], kb * kTileK, tile * 128, pol);
-        }
+        ptx::mbar_expect_tx(&full_bar[npre], w_bytes);
+        tc_load_w<EPI>(smem + (size_t)npre * p.stage_bytes, &tw, &full_bar[npre], p, tile, kb, pol);
       }
     }
   }
@@ -113,9 +106,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (warp == 1) ptx::tmem_dealloc(tmem_base, p.tmem_cols);
     return;
   }
-  const int BN = max(16, (m + 15) & ~15);
-  const uint32_t x_bytes = (SPLIT ? 2u : 1u) * (uint32_t)BN * 128u;
-  const uint32_t lo_off = kTileABytes + (uint32_t)p.bn_max * 128u;   // B_lo tile offset in a stage
+  const uint32_t x_bytes = tc_x_bytes(m, SPLIT);
+  const uint32_t acc_cols = (uint32_t)(p.mt * p.bw);
 
   if (warp == 0) {
     // ------------------------------------------------------------------ TMA
@@ -128,29 +120,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int tile = u % p.n_tiles, split = u / p.n_tiles;
         const int kb0 = split * p.kb_per_split, kb1 = min(p.kb_total, kb0 + p.kb_per_split);
         for (int kb = kb0; kb < kb1; ++kb) {
-          uint8_t* a = smem + (size_t)stage * p.stage_bytes;
-          uint8_t* b = a + kTileABytes;
+          uint8_t* st = smem + (size_t)stage * p.stage_bytes;
           if (issued < npre) {
-            // weight tile already in flight: add the activation tile
+            // weight tile already in flight: add the activation tiles
             ptx::mbar_arrive_expect_tx(&full_bar[stage], x_bytes);
           } else {
             if (!ptx::mbar_wait_bounded(&empty_bar[stage], ph ^ 1u, kWaitLimitNs, &abort_flag)) {
               ok = false;
               break;
             }
-            ptx::mbar_arrive_expect_tx(&full_bar[stage], kTileABytes + x_bytes);
-            if (EPI == EPI_SWIGLU) {
-              ptx::tma_load_2d_hint(a, &tw, &full_bar[stage], kb * kTileK, tile * 64, pol);
-              ptx::tma_load_2d_hint(a + kTileABytes / 2, &tw, &full_bar[stage], kb * kTileK, p.N + tile * 64,
-                                    pol);
-            } else {
-              ptx::tma_load_2d_hint(a, &tw, &full_bar[stage], kb * kTileK, tile * 128, pol);
-            }
+            ptx::mbar_arrive_expect_tx(&full_bar[stage], w_bytes + x_bytes);
+            tc_load_w<EPI>(st, &tw, &full_bar[stage], p, tile, kb, pol);
           }
-          for (int r = 0; r < BN / 16; ++r) {
-            ptx::tma_load_2d(b + r * 2048, &tx, &full_bar[stage], kb * kTileK, r * 16);
-            if (SPLIT) ptx::tma_load_2d(a + lo_off + r * 2048, &txlo, &full_bar[stage], kb * kTileK, r * 16);
-          }
+          tc_load_x<SPLIT>(st, &tx, &txlo, &full_bar[stage], p, m, kb);
           ++issued;
           if (++stage == p.stages) {
             stage = 0;
@@ -168,7 +150,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------------ MMA
     if (lane == 0) {
-      const uint32_t idesc = ptx::idesc_bf16_m128((uint32_t)BN);
+      const uint32_t idesc = ptx::idesc_bf16(128u, (uint32_t)p.bw);
       int stage = 0;
       uint32_t ph = 0;
       int acc = 0;
@@ -180,7 +162,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int kb0 = split * p.kb_per_split, kb1 = min(p.kb_total, kb0 + p.kb_per_split);
         if (!ptx::mbar_wait_bounded(&tempty_bar[acc], acc_ph ^ 1u, kWaitLimitNs, &abort_flag)) break;
         ptx::tc_fence_after();
-        const uint32_t d = tmem_base + (uint32_t)(acc * p.bn_max);
+        const uint32_t d = tmem_base + (uint32_t)acc * acc_cols;
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!ptx::mbar_wait_bounded(&full_bar[stage], ph, kWaitLimitNs, &abort_flag)) {
             ok = false;
@@ -188,17 +170,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           }
           consumed = ++n_consumed;
           ptx::tc_fence_after();
-          const uint8_t* a = smem + (size_t)stage * p.stage_bytes;
-          const uint64_t da = ptx::smem_desc_sw128(a);
-          const uint64_t db = ptx::smem_desc_sw128(a + kTileABytes);
-#pragma unroll
-          for (int k = 0; k < kTileK / 16; ++k) {
-            ptx::mma_bf16(d, da + 2ull * k, db + 2ull * k, idesc, (kb > kb0 || k > 0) ? 1u : 0u);
-            if (SPLIT) {
-              const uint64_t dl = ptx::smem_desc_sw128(a + lo_off);
-              ptx::mma_bf16(d, da + 2ull * k, dl + 2ull * k, idesc, 1u);
-            }
-          }
+          tc_mma_stage<SPLIT>(smem + (size_t)stage * p.stage_bytes, d, p, m, idesc, kb == kb0);
           ptx::mma_commit(&empty_bar[stage]);
           if (++stage == p.stages) {
             stage = 0;
@@ -207,8 +179,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         if (!ok) break;
         ptx::mma_commit(&tfull_bar[acc]);
-        acc ^= 1;
-        if (acc == 0) acc_ph ^= 1u;
+        if (p.acc_bufs == 2) {
+          acc ^= 1;
+          if (acc == 0) acc_ph ^= 1u;
+        } else {
+          acc_ph ^= 1u;
+        }
       }
       // all issued MMAs complete before TMEM is released
       ptx::mma_commit(&done_bar);
@@ -218,71 +194,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     __syncwarp();
   } else {
     // ------------------------------------------------------------- epilogue
-    const int lane_base = (warp & 3) * 32;
-    const int row = lane_base + lane;
     int acc = 0;
     uint32_t acc_ph = 0;
     for (int u = blockIdx.x; u < p.units; u += gridDim.x) {
-      const int tile = u % p.n_tiles, split = u / p.n_tiles;
       const bool ok = ptx::mbar_wait_bounded(&tfull_bar[acc], acc_ph, kWaitLimitNs, &abort_flag);
       if (epi_bar_any(!ok)) break;
       ptx::tc_fence_after();
-      const uint32_t taddr = tmem_base + ((uint32_t)lane_base << 16) + (uint32_t)(acc * p.bn_max);
-      float v[16];
-      if (p.splits == 1) {
-        for (int c0 = 0; c0 < BN; c0 += 16) {
-          ptx::tmem_ld16(taddr + c0, v);
-          apply_epilogue<EPI, SPLIT>(p, tile, row, c0, m, v, xch);
-        }
-        ptx::tc_fence_before();
-        if (lane == 0) ptx::mbar_arrive(&tempty_bar[acc]);
+      tc_epilogue_unit<EPI, SPLIT>(p, u, m, tmem_base + (uint32_t)acc * acc_cols, &tempty_bar[acc], &last_flag);
+      if (p.acc_bufs == 2) {
+        acc ^= 1;
+        if (acc == 0) acc_ph ^= 1u;
       } else {
-        float* slot = p.ws + (size_t)u * p.bn_max * 128;
-        for (int c0 = 0; c0 < BN; c0 += 16) {
-          ptx::tmem_ld16(taddr + c0, v);
-#pragma unroll
-          for (int i = 0; i < 16; ++i)
-            if (c0 + i < m) __stcg(slot + (size_t)(c0 + i) * 128 + row, v[i]);
-        }
-        ptx::tc_fence_before();
-        if (lane == 0) ptx::mbar_arrive(&tempty_bar[acc]);
-        epi_bar();
-        if (threadIdx.x == 64) {
-          __threadfence();
-          const int old = atomicAdd(&p.ctr[tile], 1);
-          last_flag = (old == p.splits - 1);
-          if (last_flag) p.ctr[tile] = 0;
-          __threadfence();
-        }
-        epi_bar();
-        if (last_flag) {
-          __threadfence();
-          for (int c0 = 0; c0 < BN; c0 += 16) {
-            const int nc = min(16, m - c0);
-#pragma unroll
-            for (int i = 0; i < 16; ++i) v[i] = 0.f;
-            // four splits' loads in flight per round, summed in split order
-            for (int s = 0; s < p.splits; s += 4) {
-              float t[4][16];
-#pragma unroll
-              for (int q = 0; q < 4; ++q) {
-                const float* sl = p.ws + (size_t)((s + q) * p.n_tiles + tile) * p.bn_max * 128 + row;
-#pragma unroll
-                for (int i = 0; i < 16; ++i)
-                  t[q][i] = (s + q < p.splits && i < nc) ? __ldcg(sl + (size_t)(c0 + i) * 128) : 0.f;
-              }
-#pragma unroll
-              for (int q = 0; q < 4; ++q)
-#pragma unroll
-                for (int i = 0; i < 16; ++i) v[i] += t[q][i];
-            }
-            apply_epilogue<EPI, SPLIT>(p, tile, row, c0, m, v, xch);
-          }
-        }
-        epi_bar();
+        acc_ph ^= 1u;
       }
-      acc ^= 1;
-      if (acc == 0) acc_ph ^= 1u;
     }
   }
 
@@ -326,29 +250,37 @@ static bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t K
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Split-K factor: the smallest one whose last wave of persistent CTAs is at
-// least 80% busy (every split >= 4 K-blocks); fewer splits mean fewer
-// per-unit epilogues and partial sums.  Falls back to the best efficiency.
+// Split-K factor.  Every SM streams at most its share of HBM bandwidth, so
+// the units (tile, split) should keep all SMs busy: among the factors whose
+// persistent waves are at least 90% occupied (every split >= 4 K blocks, none
+// empty), the one with the fewest waves, then the fewest splits; otherwise the
+// best occupancy.
 static int choose_splits(int tiles, int kb, int sms) {
-  int best = 1;
+  int best = 1, best_waves = 1 << 30;
   double best_eff = -1.0;
-  for (int s = 1; s <= 32; ++s) {
+  int fb = 1;
+  double fb_eff = -1.0;
+  for (int s = 1; s <= 16; ++s) {
     const int kps = (kb + s - 1) / s;
     if (s > 1 && (kps < 4 || (s - 1) * kps >= kb)) continue;
     const int units = tiles * s;
     const int waves = (units + sms - 1) / sms;
     const double eff = (double)units / (double)(waves * sms);
-    if (eff >= 0.8) return s;
-    if (eff > best_eff + 0.02) {
-      best_eff = eff;
+    if (eff >= 0.9 && waves < best_waves) {
       best = s;
+      best_waves = waves;
+      best_eff = eff;
+    }
+    if (eff > fb_eff + 0.02) {
+      fb_eff = eff;
+      fb = s;
     }
   }
-  return best;
+  return best_eff > 0 ? best : fb;
 }
 
 bool gemm_tc_supported(const Ctx& c) {
-  if (c.dtype != BUDDY_DTYPE_BF16 || c.maxB > 256) return false;
+  if (c.dtype != BUDDY_DTYPE_BF16 || c.maxB > 256 || (c.hd != 64 && c.hd != 128)) return false;
   const char* env = getenv("BUDDY_GEMM");
   if (env && env[0] == 's') return false;   // "simt": CUDA-core kernel for every GEMM
   int major = 0, minor = 0;
@@ -361,17 +293,29 @@ int gemm_tc_prepare(Ctx& c) {
   c.use_tc = gemm_tc_supported(c);
   c.use_lk = false;
   if (!c.use_tc) return BUDDY_OK;
-  c.tc_bn_max = std::max(16, (c.maxB + 15) & ~15);
-  const int smem_limit = 227 * 1024 - 12 * 1024;  // leave room for static shared memory (~9.5 KiB)
+  // geometry: 256 weight rows per tile; one M-tile per 128 rows of the batch
+  c.tc_bw = kTileN;
+  c.tc_mt = c.maxB > 128 ? 2 : 1;
+  c.tc_rows_max = std::max(16, (c.maxB + 15) & ~15);
+  c.tc_xr = c.tc_mt == 1 ? (uint32_t)c.tc_rows_max * 128u : kXTileMax;
+  // One CTA per SM with the full ring; optionally (BUDDY_TC_DUAL=1) two CTAs
+  // per SM with a short ring and one accumulator, where at least two stages
+  // fit in half of the shared memory (measured slower on the 8B decode chain).
+  const int full_limit = 227 * 1024 - 2 * 1024;   // room for static shared memory
+  const int half_limit = 111 * 1024;
+  const uint32_t sb_max = (uint32_t)c.tc_bw * 128u + 2u * c.tc_mt * c.tc_xr;
+  const char* dual_env = getenv("BUDDY_TC_DUAL");
+  c.tc_dual = dual_env && dual_env[0] == '1' && (int)((half_limit - 1024) / sb_max) >= 2;
+  c.tc_acc_bufs = c.tc_dual || c.tc_mt == 2 ? 1 : 2;
+  c.tc_tmem_cols = c.tc_dual ? 256 : 512;
+  const int limit = c.tc_dual ? half_limit : full_limit;
   for (int v = 0; v < 2; ++v) {
-    const uint32_t stage_bytes = kTileABytes + (uint32_t)(v + 1) * (uint32_t)c.tc_bn_max * 128u;
-    c.tc_stages[v] = std::min(kTcMaxStages, (int)((smem_limit - 1024) / stage_bytes));
+    const uint32_t stage_bytes = (uint32_t)c.tc_bw * 128u + (uint32_t)(v + 1) * c.tc_mt * c.tc_xr;
+    c.tc_stages[v] = std::min(kTcMaxStages, (int)((limit - 1024) / stage_bytes));
     c.tc_stage_bytes[v] = stage_bytes;
+    c.tc_w_off[v] = (uint32_t)(v + 1) * c.tc_mt * c.tc_xr;
     c.tc_smem[v] = c.tc_stages[v] * stage_bytes + 1024;
   }
-  uint32_t cols = 32;
-  while (cols < 2u * (uint32_t)c.tc_bn_max) cols <<= 1;
-  c.tc_tmem_cols = cols;
   size_t ws = 0;
   int max_tiles = 1;
   for (int w = 0; w < 4; ++w) {
@@ -380,7 +324,8 @@ int gemm_tc_prepare(Ctx& c) {
     const int kb = (K + kTileK - 1) / kTileK;
     c.tc_splits[w] = choose_splits(tiles, kb, c.num_sms);
     c.tc_tiles[w] = tiles;
-    if (c.tc_splits[w] > 1) ws = std::max(ws, (size_t)tiles * c.tc_splits[w] * c.tc_bn_max * 128);
+    // every unit stages its accumulator rows in the workspace
+    ws = std::max(ws, (size_t)tiles * c.tc_splits[w] * c.tc_rows_max * c.tc_bw);
     max_tiles = std::max(max_tiles, tiles);
   }
   // tensor maps: activations (fixed scratch) and per-layer weights
@@ -393,8 +338,9 @@ int gemm_tc_prepare(Ctx& c) {
   for (int l = 0; l < c.L; ++l) {
     const buddy_layer_weights& w = c.layers[l];
     CUtensorMap* M = &c.tmaps_host[(size_t)l * 4];
-    if (!make_map(&M[0], w.w_qkv, c.qkvN, c.d, 128) || !make_map(&M[1], w.w_o, c.d, c.qd, 128) ||
-        !make_map(&M[2], w.w_gate_up, 2ull * c.F, c.d, 64) || !make_map(&M[3], w.w_down, c.d, c.F, 128))
+    const uint32_t bw = (uint32_t)c.tc_bw;
+    if (!make_map(&M[0], w.w_qkv, c.qkvN, c.d, bw) || !make_map(&M[1], w.w_o, c.d, c.qd, bw) ||
+        !make_map(&M[2], w.w_gate_up, 2ull * c.F, c.d, bw / 2) || !make_map(&M[3], w.w_down, c.d, c.F, bw))
       return BUDDY_ERR_ARG;
   }
   if (ws > c.gemm_ws_elems) {
@@ -441,10 +387,15 @@ void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s) {
   p.splits = c.tc_splits[which];
   p.kb_per_split = (p.kb_total + p.splits - 1) / p.splits;
   p.units = tiles * p.splits;
-  p.bn_max = c.tc_bn_max;
+  p.bw = c.tc_bw;
+  p.mt = c.tc_mt;
+  p.rows_max = c.tc_rows_max;
   const int v = a.split ? 1 : 0;
   p.stages = c.tc_stages[v];
+  p.acc_bufs = c.tc_acc_bufs;
   p.stage_bytes = c.tc_stage_bytes[v];
+  p.xr = c.tc_xr;
+  p.w_off = c.tc_w_off[v];
   p.tmem_cols = c.tc_tmem_cols;
   p.rows = a.sel.rows;
   p.count = a.sel.count;

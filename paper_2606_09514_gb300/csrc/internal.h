@@ -165,8 +165,10 @@ struct Ctx {
   // tcgen05 GEMM resources
   bool use_tc = false;
   std::vector<CUtensorMap> tmaps_host;    // per layer 4 weight maps, then 3 activation maps
-  int tc_bn_max = 16, tc_stages[2] = {1, 1}, tc_smem[2] = {0, 0};   // [plain, split activations]
-  uint32_t tc_stage_bytes[2] = {0, 0}, tc_tmem_cols = 32;
+  int tc_bw = 256, tc_mt = 1, tc_rows_max = 16, tc_acc_bufs = 2;   // tile geometry (gemm_common.cuh)
+  int tc_stages[2] = {1, 1}, tc_smem[2] = {0, 0};                   // [plain, split activations]
+  uint32_t tc_stage_bytes[2] = {0, 0}, tc_w_off[2] = {0, 0}, tc_xr = 0, tc_tmem_cols = 512;
+  bool tc_dual = false;                   // two GEMM CTAs per SM (short ring, one accumulator)
   int tc_splits[4] = {1, 1, 1, 1}, tc_tiles[4] = {1, 1, 1, 1};
   bool use_lk = false;                    // per-layer persistent kernel (small batches)
   unsigned* lk_bar = nullptr;             // its grid barrier [arrivals, generation]

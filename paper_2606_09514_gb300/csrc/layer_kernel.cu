@@ -32,10 +32,6 @@ namespace buddy {
 
 constexpr int kLkThreads = 192;
 
-struct LkGemm {
-  int N, K, n_tiles, splits, kb_total, kb_per_split, units;
-};
-
 struct LkMaps {
   CUtensorMap w[4];     // qkv, o, gate_up, down weights
   CUtensorMap x[4];     // activation operand of each GEMM (xn, attn, xn, act)
@@ -54,11 +50,9 @@ struct LkParams {
   int d;
   bf16* xn;
   bf16* xn_lo;
-  LkGemm g[4];
   int stages;
   uint32_t stage_bytes;
   uint32_t tmem_cols;
-  int bn_max;
   uint32_t attn_off;     // byte offset of the attention region in dynamic shared memory
   unsigned* bar;         // grid barrier: [0] arrivals, [1] generation
   TcParams tp[4];        // epilogue parameters of each GEMM
@@ -138,74 +132,18 @@ __device__ __forceinline__ void lk_norm(const LkParams& p, const float* X, const
   }
 }
 
-// Drains this CTA's units of GEMM `ph` from TMEM and applies its epilogue
-// (directly, or through the deterministic split-K fixup).
+// Drains this CTA's units of GEMM `ph` from TMEM and applies its epilogue.
 template <int EPI, bool SPLIT>
-__device__ __forceinline__ bool lk_epilogue(const LkParams& p, int ph, int m, int BN, uint32_t tmem_base,
+__device__ __forceinline__ bool lk_epilogue(const LkParams& p, int ph, int m, uint32_t tmem_base,
                                             uint64_t* tfull_bar, uint64_t* tempty_bar, int& acc, uint32_t& acc_ph,
-                                            volatile int* abort_flag, float* xch, int* last_flag) {
+                                            volatile int* abort_flag, int* last_flag) {
   const TcParams& tp = p.tp[ph];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int lane_base = (warp & 3) * 32;
-  const int row = lane_base + lane;
-  for (int u = blockIdx.x; u < p.g[ph].units; u += gridDim.x) {
-    const int tile = u % p.g[ph].n_tiles;
+  const uint32_t acc_cols = (uint32_t)(tp.mt * tp.bw);
+  for (int u = blockIdx.x; u < tp.units; u += gridDim.x) {
     const bool ok = ptx::mbar_wait_bounded(&tfull_bar[acc], acc_ph, kWaitLimitNs, abort_flag);
     if (epi_bar_any(!ok)) return false;
     ptx::tc_fence_after();
-    const uint32_t taddr = tmem_base + ((uint32_t)lane_base << 16) + (uint32_t)(acc * p.bn_max);
-    float v[16];
-    if (tp.splits == 1) {
-      for (int c0 = 0; c0 < BN; c0 += 16) {
-        ptx::tmem_ld16(taddr + c0, v);
-        apply_epilogue<EPI, SPLIT>(tp, tile, row, c0, m, v, xch);
-      }
-      ptx::tc_fence_before();
-      if (lane == 0) ptx::mbar_arrive(&tempty_bar[acc]);
-    } else {
-      float* slot = tp.ws + (size_t)u * p.bn_max * 128;
-      for (int c0 = 0; c0 < BN; c0 += 16) {
-        ptx::tmem_ld16(taddr + c0, v);
-#pragma unroll
-        for (int i = 0; i < 16; ++i)
-          if (c0 + i < m) __stcg(slot + (size_t)(c0 + i) * 128 + row, v[i]);
-      }
-      ptx::tc_fence_before();
-      if (lane == 0) ptx::mbar_arrive(&tempty_bar[acc]);
-      epi_bar();
-      if (threadIdx.x == 64) {
-        __threadfence();
-        const int old = atomicAdd(&tp.ctr[tile], 1);
-        *last_flag = (old == tp.splits - 1);
-        if (*last_flag) tp.ctr[tile] = 0;
-        __threadfence();
-      }
-      epi_bar();
-      if (*last_flag) {
-        __threadfence();
-        for (int c0 = 0; c0 < BN; c0 += 16) {
-          const int nc = min(16, m - c0);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) v[i] = 0.f;
-          for (int s = 0; s < tp.splits; s += 4) {
-            float tt[4][16];
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              const float* sl = tp.ws + (size_t)((s + q) * tp.n_tiles + tile) * p.bn_max * 128 + row;
-#pragma unroll
-              for (int i = 0; i < 16; ++i)
-                tt[q][i] = (s + q < tp.splits && i < nc) ? __ldcg(sl + (size_t)(c0 + i) * 128) : 0.f;
-            }
-#pragma unroll
-            for (int q = 0; q < 4; ++q)
-#pragma unroll
-              for (int i = 0; i < 16; ++i) v[i] += tt[q][i];
-          }
-          apply_epilogue<EPI, SPLIT>(tp, tile, row, c0, m, v, xch);
-        }
-      }
-      epi_bar();
-    }
+    tc_epilogue_unit<EPI, SPLIT>(tp, u, m, tmem_base + (uint32_t)acc * acc_cols, &tempty_bar[acc], last_flag);
     acc ^= 1;
     if (acc == 0) acc_ph ^= 1u;
   }
@@ -221,13 +159,11 @@ __global__ void __launch_bounds__(kLkThreads, 1)
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag, passed, ok_s, consumed;
   __shared__ int last_flag;
-  __shared__ float xch[128 * 17];
   __shared__ float red[64], inv[16], sc[32];
 
   if (call_aborted(p.status)) return;
   const int m = p.count ? *p.count : p.n;
   if (m <= 0) return;
-  const int BN = max(16, (m + 15) & ~15);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
 
@@ -255,8 +191,8 @@ __global__ void __launch_bounds__(kLkThreads, 1)
   __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem_base = tmem_slot;
-  const uint32_t x_bytes = (SPLIT ? 2u : 1u) * (uint32_t)BN * 128u;
-  const uint32_t lo_off = kTileABytes + (uint32_t)p.bn_max * 128u;
+  const uint32_t x_bytes = tc_x_bytes(m, SPLIT);
+  const uint32_t w_bytes = (uint32_t)p.tp[0].bw * 128u;
 
   if (warp == 0) {
     // --------------------------------------------------------- TMA producer
@@ -267,12 +203,9 @@ __global__ void __launch_bounds__(kLkThreads, 1)
       auto flush = [&]() {
         while (ph_cnt > 0 && passed >= x_ready(pend_ph[ph_head])) {
           const int s = pend_stage[ph_head], ph = pend_ph[ph_head], kb = pend_kb[ph_head];
-          uint8_t* a = smem + (size_t)s * p.stage_bytes;
           ptx::mbar_arrive_expect_tx(&full_bar[s], x_bytes);
-          for (int r = 0; r < BN / 16; ++r) {
-            ptx::tma_load_2d(a + kTileABytes + r * 2048, &maps.x[ph], &full_bar[s], kb * kTileK, r * 16);
-            if (SPLIT) ptx::tma_load_2d(a + lo_off + r * 2048, &maps.xlo[ph], &full_bar[s], kb * kTileK, r * 16);
-          }
+          tc_load_x<SPLIT>(smem + (size_t)s * p.stage_bytes, &maps.x[ph], &maps.xlo[ph], &full_bar[s], p.tp[ph], m,
+                           kb);
           ph_head = (ph_head + 1) % kTcMaxStages;
           --ph_cnt;
         }
@@ -281,7 +214,7 @@ __global__ void __launch_bounds__(kLkThreads, 1)
       uint32_t ph_bit = 0;
       bool ok = true;
       for (int ph = 0; ph < 4 && ok; ++ph) {
-        const LkGemm& G = p.g[ph];
+        const TcParams& G = p.tp[ph];
         for (int u = blockIdx.x; u < G.units && ok; u += gridDim.x) {
           const int tile = u % G.n_tiles, split = u / G.n_tiles;
           const int kb0 = split * G.kb_per_split, kb1 = min(G.kb_total, kb0 + G.kb_per_split);
@@ -299,20 +232,24 @@ __global__ void __launch_bounds__(kLkThreads, 1)
             }
             if (!ok) break;
             uint8_t* a = smem + (size_t)stage * p.stage_bytes;
-            ptx::mbar_expect_tx(&full_bar[stage], kTileABytes);
-            if (ph == 2) {
-              ptx::tma_load_2d_hint(a, &maps.w[2], &full_bar[stage], kb * kTileK, tile * 64, pol);
-              ptx::tma_load_2d_hint(a + kTileABytes / 2, &maps.w[2], &full_bar[stage], kb * kTileK,
-                                    G.N + tile * 64, pol);
+            // activations already available (no earlier stage waiting): one
+            // arrival covers both tiles; otherwise the activation tile waits
+            // in the queue for its barrier
+            const bool x_now = ph_cnt == 0 && passed >= x_ready(ph);
+            if (x_now) ptx::mbar_arrive_expect_tx(&full_bar[stage], w_bytes + x_bytes);
+            else ptx::mbar_expect_tx(&full_bar[stage], w_bytes);
+            if (ph == 2) tc_load_w<EPI_SWIGLU>(a, &maps.w[2], &full_bar[stage], G, tile, kb, pol);
+            else tc_load_w<EPI_RESID>(a, &maps.w[ph], &full_bar[stage], G, tile, kb, pol);
+            if (x_now) {
+              tc_load_x<SPLIT>(a, &maps.x[ph], &maps.xlo[ph], &full_bar[stage], G, m, kb);
             } else {
-              ptx::tma_load_2d_hint(a, &maps.w[ph], &full_bar[stage], kb * kTileK, tile * 128, pol);
+              const int slot = (ph_head + ph_cnt) % kTcMaxStages;
+              pend_stage[slot] = stage;
+              pend_ph[slot] = ph;
+              pend_kb[slot] = kb;
+              ++ph_cnt;
+              flush();
             }
-            const int slot = (ph_head + ph_cnt) % kTcMaxStages;
-            pend_stage[slot] = stage;
-            pend_ph[slot] = ph;
-            pend_kb[slot] = kb;
-            ++ph_cnt;
-            flush();
             ++issued;
             if (++stage == p.stages) {
               stage = 0;
@@ -342,12 +279,12 @@ __global__ void __launch_bounds__(kLkThreads, 1)
   } else if (warp == 1) {
     // -------------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      const uint32_t idesc = ptx::idesc_bf16_m128((uint32_t)BN);
+      const uint32_t idesc = ptx::idesc_bf16(128u, (uint32_t)p.tp[0].bw);
       int stage = 0, acc = 0, n_consumed = 0;
       uint32_t ph_bit = 0, acc_ph = 0;
       bool ok = true;
       for (int ph = 0; ph < 4 && ok; ++ph) {
-        const LkGemm& G = p.g[ph];
+        const TcParams& G = p.tp[ph];
         for (int u = blockIdx.x; u < G.units && ok; u += gridDim.x) {
           const int split = u / G.n_tiles;
           const int kb0 = split * G.kb_per_split, kb1 = min(G.kb_total, kb0 + G.kb_per_split);
@@ -356,7 +293,7 @@ __global__ void __launch_bounds__(kLkThreads, 1)
             break;
           }
           ptx::tc_fence_after();
-          const uint32_t dcol = tmem_base + (uint32_t)(acc * p.bn_max);
+          const uint32_t dcol = tmem_base + (uint32_t)(acc * G.mt * G.bw);
           for (int kb = kb0; kb < kb1; ++kb) {
             if (!ptx::mbar_wait_bounded(&full_bar[stage], ph_bit, kWaitLimitNs, &abort_flag)) {
               ok = false;
@@ -364,15 +301,7 @@ __global__ void __launch_bounds__(kLkThreads, 1)
             }
             consumed = ++n_consumed;
             ptx::tc_fence_after();
-            const uint8_t* a = smem + (size_t)stage * p.stage_bytes;
-            const uint64_t da = ptx::smem_desc_sw128(a);
-            const uint64_t db = ptx::smem_desc_sw128(a + kTileABytes);
-            const uint64_t dl = ptx::smem_desc_sw128(a + lo_off);
-#pragma unroll
-            for (int k = 0; k < kTileK / 16; ++k) {
-              ptx::mma_bf16(dcol, da + 2ull * k, db + 2ull * k, idesc, (kb > kb0 || k > 0) ? 1u : 0u);
-              if (SPLIT) ptx::mma_bf16(dcol, da + 2ull * k, dl + 2ull * k, idesc, 1u);
-            }
+            tc_mma_stage<SPLIT>(smem + (size_t)stage * p.stage_bytes, dcol, G, m, idesc, kb == kb0);
             ptx::mma_commit(&empty_bar[stage]);
             if (++stage == p.stages) {
               stage = 0;
@@ -399,25 +328,25 @@ __global__ void __launch_bounds__(kLkThreads, 1)
     bool ok = true;
     lk_norm<SPLIT>(p, p.src, p.g1, m, t, red, inv);
     ok = lk_grid_sync(p.bar, gen, &abort_flag, &passed, &ok_s, p.status);                          // B1
-    if (ok) ok = lk_epilogue<EPI_QKV, SPLIT>(p, 0, m, BN, tmem_base, tfull_bar, tempty_bar, acc, acc_ph,
-                                            &abort_flag, xch, &last_flag);
+    if (ok) ok = lk_epilogue<EPI_QKV, SPLIT>(p, 0, m, tmem_base, tfull_bar, tempty_bar, acc, acc_ph, &abort_flag,
+                                              &last_flag);
     if (ok) ok = lk_grid_sync(p.bar, gen, &abort_flag, &passed, &ok_s, p.status);                  // B2
     if (ok) {
       attn_run<bf16, 128>(p.attn, t, blockIdx.x, gridDim.x, smem + p.attn_off, sc, SyncEpilogueWarps{}, false);
       ok = lk_grid_sync(p.bar, gen, &abort_flag, &passed, &ok_s, p.status);                        // B3
     }
-    if (ok) ok = lk_epilogue<EPI_RESID, SPLIT>(p, 1, m, BN, tmem_base, tfull_bar, tempty_bar, acc, acc_ph,
-                                              &abort_flag, xch, &last_flag);
+    if (ok) ok = lk_epilogue<EPI_RESID, SPLIT>(p, 1, m, tmem_base, tfull_bar, tempty_bar, acc, acc_ph, &abort_flag,
+                                              &last_flag);
     if (ok) ok = lk_grid_sync(p.bar, gen, &abort_flag, &passed, &ok_s, p.status);                  // B4
     if (ok) {
       lk_norm<SPLIT>(p, p.H, p.g2, m, t, red, inv);
       ok = lk_grid_sync(p.bar, gen, &abort_flag, &passed, &ok_s, p.status);                        // B5
     }
-    if (ok) ok = lk_epilogue<EPI_SWIGLU, SPLIT>(p, 2, m, BN, tmem_base, tfull_bar, tempty_bar, acc, acc_ph,
-                                               &abort_flag, xch, &last_flag);
+    if (ok) ok = lk_epilogue<EPI_SWIGLU, SPLIT>(p, 2, m, tmem_base, tfull_bar, tempty_bar, acc, acc_ph, &abort_flag,
+                                              &last_flag);
     if (ok) ok = lk_grid_sync(p.bar, gen, &abort_flag, &passed, &ok_s, p.status);                  // B6
-    if (ok) ok = lk_epilogue<EPI_RESID, SPLIT>(p, 3, m, BN, tmem_base, tfull_bar, tempty_bar, acc, acc_ph,
-                                              &abort_flag, xch, &last_flag);
+    if (ok) ok = lk_epilogue<EPI_RESID, SPLIT>(p, 3, m, tmem_base, tfull_bar, tempty_bar, acc, acc_ph, &abort_flag,
+                                              &last_flag);
     if (!ok && t == 0) abort_flag = 1;
   }
 
@@ -434,17 +363,20 @@ __global__ void __launch_bounds__(kLkThreads, 1)
 // ---------------------------------------------------------------------------
 // Host side
 // ---------------------------------------------------------------------------
+// Ring of stages followed by the attention region.
+constexpr int kLkSmemLimit = 227 * 1024 - 2 * 1024;   // room for static shared memory
+
 static int lk_smem_budget(const Ctx& c, bool split, size_t attn_bytes, int* stages, uint32_t* stage_bytes) {
-  const uint32_t sb = kTileABytes + (split ? 2u : 1u) * (uint32_t)c.tc_bn_max * 128u;
-  const int limit = 227 * 1024 - 12 * 1024;   // static shared memory ~10 KiB
-  const int avail = limit - 1024 - (int)((attn_bytes + 1023) & ~size_t(1023));
+  const uint32_t sb = c.tc_stage_bytes[split ? 1 : 0];
+  const int tail = (int)((attn_bytes + 1023) & ~size_t(1023));
+  const int avail = kLkSmemLimit - 1024 - tail;
   *stages = std::min(kTcMaxStages, avail / (int)sb);
   *stage_bytes = sb;
-  return *stages >= 3 ? (int)(*stages * sb + 1024 + ((attn_bytes + 1023) & ~size_t(1023))) : 0;
+  return *stages >= 3 ? (int)(*stages * sb + 1024 + tail) : 0;
 }
 
 bool layer_kernel_supported(const Ctx& c) {
-  return c.use_tc && c.maxB <= 16 && c.hd == 128 && c.d % 32 == 0 && c.nq / c.nkv <= 8;
+  return c.use_tc && c.tc_mt == 1 && c.maxB <= 16 && c.hd == 128 && c.d % 32 == 0 && c.nq / c.nkv <= 8;
 }
 
 // One block on the rows of `sel` with the persistent kernel.  Returns false if
@@ -461,7 +393,7 @@ bool launch_layer_kernel(const Ctx& c, const buddy_kv_state& kv, int l, RowSel s
   static bool attr_set[2] = {false, false};
   if (!attr_set[split]) {
     if (cudaFuncSetAttribute(split ? layer_kernel<true> : layer_kernel<false>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024 - 12 * 1024) != cudaSuccess)
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, kLkSmemLimit) != cudaSuccess)
       return false;
     attr_set[split] = true;
   }
@@ -478,15 +410,13 @@ bool launch_layer_kernel(const Ctx& c, const buddy_kv_state& kv, int l, RowSel s
   for (int w = 0; w < 4; ++w) {
     int N, K, tiles;
     gemm_shape(c, w, &N, &K, &tiles);
-    LkGemm& g = p.g[w];
-    g.N = N; g.K = K; g.n_tiles = tiles; g.splits = c.tc_splits[w];
-    g.kb_total = (K + kTileK - 1) / kTileK;
-    g.kb_per_split = (g.kb_total + g.splits - 1) / g.splits;
-    g.units = tiles * g.splits;
     TcParams& tp = p.tp[w];
-    tp.N = N; tp.K = K; tp.n_tiles = tiles; tp.splits = g.splits; tp.kb_total = g.kb_total;
-    tp.kb_per_split = g.kb_per_split; tp.units = g.units; tp.bn_max = c.tc_bn_max; tp.stages = stages;
-    tp.stage_bytes = stage_bytes; tp.tmem_cols = c.tc_tmem_cols;
+    tp.N = N; tp.K = K; tp.n_tiles = tiles; tp.splits = c.tc_splits[w];
+    tp.kb_total = (K + kTileK - 1) / kTileK;
+    tp.kb_per_split = (tp.kb_total + tp.splits - 1) / tp.splits;
+    tp.units = tiles * tp.splits;
+    tp.bw = c.tc_bw; tp.mt = c.tc_mt; tp.rows_max = c.tc_rows_max; tp.stages = stages; tp.acc_bufs = 2;
+    tp.stage_bytes = stage_bytes; tp.xr = c.tc_xr; tp.w_off = c.tc_w_off[split ? 1 : 0]; tp.tmem_cols = 512;
     tp.rows = sel.rows; tp.count = sel.count; tp.n = sel.n;
     tp.ws = c.gemm_ws; tp.ctr = c.gemm_ctr; tp.status = c.status;
   }
@@ -497,7 +427,7 @@ bool launch_layer_kernel(const Ctx& c, const buddy_kv_state& kv, int l, RowSel s
   p.tp[1].resid_src = src; p.tp[1].resid_dst = H;
   p.tp[2].out_act = (bf16*)c.act; p.tp[2].out_act_lo = split ? (bf16*)c.act_lo : nullptr;
   p.tp[3].resid_src = H; p.tp[3].resid_dst = H;
-  p.stages = stages; p.stage_bytes = stage_bytes; p.tmem_cols = c.tc_tmem_cols; p.bn_max = c.tc_bn_max;
+  p.stages = stages; p.stage_bytes = stage_bytes; p.tmem_cols = 512;   // one CTA per SM, two accumulators
   p.attn_off = (uint32_t)(stages * stage_bytes);
   p.bar = c.lk_bar;
   p.attn = AttnArgs<bf16>{c.q, sel.rows, sel.count, sel.n, c.nq, c.nkv, kv.len, kv.seq_off, kv.cap,
