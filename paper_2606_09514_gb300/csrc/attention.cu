@@ -24,14 +24,14 @@
 
 namespace buddy {
 
-template <typename T, int HD>
+template <typename T, int HD, int GP>
 __global__ void __launch_bounds__(kAttnThreads) attn_kernel(AttnArgs<T> A) {
   extern __shared__ __align__(16) uint8_t smraw[];
   __shared__ float sc[32];
-  attn_run<T, HD>(A, threadIdx.x, blockIdx.x, gridDim.x, smraw, sc, SyncCta{}, true);
+  attn_run<T, HD, GP>(A, threadIdx.x, blockIdx.x, gridDim.x, smraw, sc, SyncCta{}, true);
 }
 
-template <typename T, int HD>
+template <typename T, int HD, int GP>
 static void attn_impl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q,
                       void* out, void* out_lo, cudaStream_t s) {
   const int G = c.nq / c.nkv;
@@ -40,11 +40,12 @@ static void attn_impl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int la
   static int occ = 0;
   static size_t occ_smem = 0;
   if (!attr_set) {
-    cudaFuncSetAttribute(attn_kernel<T, HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+    cudaFuncSetAttribute(attn_kernel<T, HD, GP>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
     attr_set = true;
   }
   if (occ == 0 || occ_smem != smem) {   // resident CTAs per SM at this shared-memory size
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, attn_kernel<T, HD>, kAttnThreads, smem) != cudaSuccess)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, attn_kernel<T, HD, GP>, kAttnThreads, smem) !=
+        cudaSuccess)
       occ = 1;
     occ_smem = smem;
   }
@@ -52,7 +53,18 @@ static void attn_impl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int la
   AttnArgs<T> A{q, sel.rows, sel.count, sel.n, c.nq, c.nkv, kv.len, kv.seq_off, kv.cap,
                 (const T*)kv.k_cache[layer], (const T*)kv.v_cache[layer], c.attn_max_chunks, c.attn_m, c.attn_l,
                 c.attn_acc, c.attn_ctr, (T*)out, (T*)out_lo, c.status};
-  launch_k(attn_kernel<T, HD>, grid, kAttnThreads, smem, s, c.pdl, A);
+  launch_k(attn_kernel<T, HD, GP>, grid, kAttnThreads, smem, s, c.pdl, A);
+}
+
+template <typename T, int HD>
+static void attn_group(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q, void* out,
+                       void* out_lo, cudaStream_t s) {
+  switch (attn_group_pad(c.nq / c.nkv)) {
+    case 1: attn_impl<T, HD, 1>(c, sel, kv, layer, q, out, out_lo, s); break;
+    case 2: attn_impl<T, HD, 2>(c, sel, kv, layer, q, out, out_lo, s); break;
+    case 4: attn_impl<T, HD, 4>(c, sel, kv, layer, q, out, out_lo, s); break;
+    default: attn_impl<T, HD, 8>(c, sel, kv, layer, q, out, out_lo, s);
+  }
 }
 
 // Spans are at least one chunk long, so the partial buffers hold
@@ -62,11 +74,11 @@ int attention_chunk() { return kChunk; }
 void launch_attention(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q,
                       void* out, void* out_lo, cudaStream_t s) {
   if (c.dtype == BUDDY_DTYPE_BF16) {
-    if (c.hd == 128) attn_impl<bf16, 128>(c, sel, kv, layer, q, out, out_lo, s);
-    else attn_impl<bf16, 64>(c, sel, kv, layer, q, out, out_lo, s);
+    if (c.hd == 128) attn_group<bf16, 128>(c, sel, kv, layer, q, out, out_lo, s);
+    else attn_group<bf16, 64>(c, sel, kv, layer, q, out, out_lo, s);
   } else {
-    if (c.hd == 128) attn_impl<float, 128>(c, sel, kv, layer, q, out, nullptr, s);
-    else attn_impl<float, 64>(c, sel, kv, layer, q, out, nullptr, s);
+    if (c.hd == 128) attn_group<float, 128>(c, sel, kv, layer, q, out, nullptr, s);
+    else attn_group<float, 64>(c, sel, kv, layer, q, out, nullptr, s);
   }
 }
 

@@ -83,23 +83,44 @@ struct AttnArgs {
   const int32_t* status;
 };
 
-// Dynamic shared memory used by attn_run (bytes).
+// Dynamic shared memory used by attn_run (bytes): double-buffered K (rows
+// padded by 16 bytes) and V chunks, the scaled queries, the logits, the
+// probabilities by position, the span-merge weights, the row prefix and the
+// rows' cache offsets, positions and head strides.
 template <typename T, int HD>
 __host__ __device__ constexpr size_t attn_smem_fixed() {
   return 2 * (size_t)kChunk * (HD + 16 / sizeof(T)) * sizeof(T) + 2 * (size_t)kChunk * HD * sizeof(T);
 }
 inline size_t attn_smem_bytes(size_t fixed, int G, int hd, int max_spans, int max_rows) {
-  return fixed + (size_t)G * hd * 4 + (size_t)G * kChunk * 4 + (size_t)G * hd * 4 + (size_t)G * max_spans * 4 +
-         (size_t)(max_rows + 1) * 4;
+  const int gp = G <= 1 ? 1 : (G <= 2 ? 2 : (G <= 4 ? 4 : 8));
+  return fixed + (size_t)gp * hd * 4 + 2 * (size_t)gp * kChunk * 4 + (size_t)gp * max_spans * 4 +
+         (size_t)(max_rows + 1) * 4 + 8 + (size_t)max_rows * 16;
 }
+
+// Query heads per KV head rounded up to 1, 2, 4 or 8 (the work-loop template).
+inline int attn_group_pad(int G) { return G <= 1 ? 1 : (G <= 2 ? 2 : (G <= 4 ? 4 : 8)); }
 
 // Processes this CTA's share (items cta, cta + ncta, ...) of one layer's
 // attention with kAttnThreads threads numbered tid; `sync` synchronises them;
 // `sc` points to 32 floats of shared scratch.  With `pdl` the copies that do
-// not depend on the preceding kernel start before waiting on it.
-template <typename T, int HD, typename Sync>
+// not depend on the preceding kernel start before waiting on it.  GP >= G is
+// the padded number of query heads per KV head.
+//
+// Thread mapping within a 64-position chunk:
+//   logits: a warp scores 16 positions (32 for one head), 32 / GP positions x GP
+//           heads per round: lane l multiplies dims HD/32 * l.. of each K row with
+//           the same dims of the queries (held in registers), and a halving
+//           butterfly over the lanes leaves the full dot product of
+//           (position l / GP, head l % GP) in lane l;
+//   P.V:    thread t owns channels 8 * (t % (HD/8)) .. +8 of every head for the
+//           positions of group t / (HD/8); its partial sums stay in registers
+//           across the chunks of the span (rescaled by the online-softmax
+//           factor) and the groups are summed once at the end of the span.
+template <typename T, int HD, int GP, typename Sync>
 __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta, int ncta, uint8_t* smem,
                                          float* sc, Sync sync, bool pdl) {
+  static_assert(GP == 1 || GP == 2 || GP == 4 || GP == 8, "GP");
+  static_assert(HD == 64 || HD == 128, "HD");
   const float* __restrict__ q = A.q;
   const int32_t* rows = A.rows;
   const int32_t* count = A.count;
@@ -122,12 +143,9 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
   // steps: the work decomposition and the first chunk's copies can start
   // before waiting on the preceding kernel (which writes q and the new
   // token's K/V at position len[i]).
-  if (*reinterpret_cast<const volatile int32_t*>(status + 1) != 0) {
-    if (pdl) pdl_wait();
-    return;
-  }
+  const int aborted = *reinterpret_cast<const volatile int32_t*>(status + 1);
   const int m = count ? *count : n;
-  if (m <= 0) {
+  if (aborted != 0 || m <= 0) {
     if (pdl) pdl_wait();
     return;
   }
@@ -135,14 +153,22 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
   constexpr int KROW = HD + PAD;
   constexpr int V16 = HD * (int)sizeof(T) / 16;  // 16-byte pieces per row
   constexpr int E16 = 16 / sizeof(T);            // elements per piece
+  constexpr int CH = HD / 8;                     // P.V channel groups of 8
+  constexpr int NPG = kAttnThreads / CH;         // P.V position groups
+  constexpr int PPG = kChunk / NPG;              // positions per group and chunk
   const int G = nq / nkv;
   T* Kb0 = reinterpret_cast<T*>(smem);                          // 2 x [kChunk][KROW]
-  T* Vb0 = Kb0 + 2 * kChunk * KROW;                              // 2 x [kChunk][HD]
-  float* qs = reinterpret_cast<float*>(Vb0 + 2 * kChunk * HD);   // [G][HD]
-  float* ps = qs + G * HD;                                       // [G][kChunk]
-  float* red = ps + G * kChunk;                                  // [G][HD] second-half sums (HD = 64)
-  float* wch = red + G * HD;                                     // [G][max_spans] merge weights
-  int* pref = reinterpret_cast<int*>(wch + G * max_spans);       // [m + 1] span prefix over rows
+  T* Vb0 = Kb0 + 2 * kChunk * KROW;                             // 2 x [kChunk][HD]
+  float* qs = reinterpret_cast<float*>(Vb0 + 2 * kChunk * HD);  // [GP][HD]
+  float* lg = qs + GP * HD;                                     // [GP][kChunk] logits
+  float* pt = lg + GP * kChunk;                                 // [kChunk][GP] probabilities
+  float* wch = pt + GP * kChunk;                                // [GP][max_spans] merge weights
+  int* pref = reinterpret_cast<int*>(wch + GP * max_spans);     // [m + 1] span prefix over rows
+  int64_t* rbase = reinterpret_cast<int64_t*>(                  // [m] cache offset of each row
+      (reinterpret_cast<uintptr_t>(pref + m + 1) + 7) & ~uintptr_t(7));
+  int* rnp = reinterpret_cast<int*>(rbase + m);                 // [m] positions (len + 1)
+  int* rhs = rnp + m;                                           // [m] head stride (cap * HD)
+  float* red = reinterpret_cast<float*>(Kb0);                   // [NPG][GP][HD], after the last chunk
   float* alpha_s = sc;        // [8]
   float* mrun_s = sc + 8;     // [8]
   float* lrun_s = sc + 16;    // [8]
@@ -150,44 +176,51 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
   int* span_s_p = reinterpret_cast<int*>(sc + 25);
 
   const int warp = tid >> 5, lane = tid & 31;
-  // total positions -> span length P (the same value in every CTA)
+  // positions per row (kept in pref[1..m]) and their total -> span length P
   if (warp == 0) {
     long long tot = 0;
-    for (int j = lane; j < m; j += 32) tot += len[rows ? rows[j] : j] + 1;
+    for (int j = lane; j < m; j += 32) {
+      const int i = rows ? rows[j] : j;
+      const int np = len[i] + 1;
+      rnp[j] = np;
+      rbase[j] = seq_off[i] * nkv * HD;
+      rhs[j] = cap[i] * HD;
+      pref[j + 1] = np;
+      tot += np;
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
-    if (lane == 0) {
-      const long long items = max(1, ncta / 2);
-      const long long want = (tot * nkv + items - 1) / items;
-      const int P = (int)min((long long)kMaxSpan, max((long long)kChunk, want));
-      *span_s_p = (P + kChunk - 1) / kChunk * kChunk;
-    }
-  }
-  sync();
-  const int P = *span_s_p;
-  if (warp == 0) {
+    __syncwarp();
+    // about one item per CTA, at least one chunk per span
+    const long long want = (tot * nkv + ncta - 1) / ncta;
+    const int P0 = (int)min((long long)kMaxSpan, max((long long)kChunk, want));
+    const int P = (P0 + kChunk - 1) / kChunk * kChunk;
     int carry = 0;
     for (int b = 0; b < m; b += 32) {
       const int j = b + lane;
       int ns = 0;
-      if (j < m) ns = (len[rows ? rows[j] : j] + 1 + P - 1) / P;
+      if (j < m) ns = (pref[j + 1] + P - 1) / P;
       int x = ns;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
         const int y = __shfl_up_sync(0xffffffffu, x, o);
         if (lane >= o) x += y;
       }
+      __syncwarp();
       if (j < m) pref[j + 1] = carry + x;
       carry += __shfl_sync(0xffffffffu, x, 31);
     }
-    if (lane == 0) pref[0] = 0;
+    if (lane == 0) {
+      pref[0] = 0;
+      *span_s_p = P;
+    }
   }
   sync();
+  const int P = *span_s_p;
   const int total = pref[m] * nkv;
   const float scale = rsqrtf((float)HD);
   bool waited = !pdl;
-  constexpr int SPLIT = kAttnThreads / HD;   // 1 for HD = 128, 2 for HD = 64
-  const int e = tid % HD, half = tid / HD;
+  const int cg = tid % CH, pg = tid / CH;                 // P.V: channel group, position group
 
   for (int item = cta; item < total; item += ncta) {
     const int g = item % nkv;
@@ -199,13 +232,13 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
       else hi = mid;
     }
     const int j = lo, sp = js - pref[j];
-    const int i = rows ? rows[j] : j;
-    const int npos = len[i] + 1;
+    const int npos = rnp[j];
     const int nsp = pref[j + 1] - pref[j];
     const int s0 = sp * P, s1 = min(npos, s0 + P);
     const int nch = (s1 - s0 + kChunk - 1) / kChunk;
-    const T* Kbase = Kc + kv_offset(seq_off, cap, i, nkv, HD, g, 0);
-    const T* Vbase = Vc + kv_offset(seq_off, cap, i, nkv, HD, g, 0);
+    const int64_t kvo = rbase[j] + (int64_t)g * rhs[j];   // kv_offset of (row j's sequence, head g, position 0)
+    const T* Kbase = Kc + kvo;
+    const T* Vbase = Vc + kvo;
 
     auto issue = [&](int c) {   // chunk c of this span into buffer c & 1
       const int p0 = s0 + c * kChunk, cnt = min(kChunk, s1 - p0);
@@ -231,14 +264,24 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
       issue(0);
     }
     const float* qj = q + (size_t)j * nq * HD + (size_t)g * G * HD;
-    for (int x = tid; x < G * HD; x += kAttnThreads) qs[x] = qj[x] * scale;
-    if (tid < G) {
+    for (int x = tid; x < GP * HD; x += kAttnThreads) qs[x] = x < G * HD ? qj[x] * scale : 0.f;
+    sync();
+    // this lane's query dims for the logits
+    constexpr int DPL = HD / 32;
+    float qr[GP][DPL];
+#pragma unroll
+    for (int h = 0; h < GP; ++h)
+#pragma unroll
+      for (int d = 0; d < DPL; ++d) qr[h][d] = qs[h * HD + lane * DPL + d];
+    if (tid < GP) {
       mrun_s[tid] = -INFINITY;
       lrun_s[tid] = 0.f;
     }
-    float acc[8];
+    float acc[GP][8];
 #pragma unroll
-    for (int h = 0; h < 8; ++h) acc[h] = 0.f;
+    for (int h = 0; h < GP; ++h)
+#pragma unroll
+      for (int k = 0; k < 8; ++k) acc[h][k] = 0.f;
 
     for (int c = 0; c < nch; ++c) {
       if (c + 1 < nch) {
@@ -251,37 +294,72 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
       const int cnt = min(kChunk, s1 - (s0 + c * kChunk));
       const T* Ks = Kb0 + (c & 1) * kChunk * KROW;
       const T* Vs = Vb0 + (c & 1) * kChunk * HD;
-      // logits: 32 consecutive pairs of a warp share the head, differ in position
-      for (int x = tid; x < G * kChunk; x += kAttnThreads) {
-        const int h = x / kChunk, p = x - h * kChunk;
-        float a = -INFINITY;
-        if (p < cnt) {
-          a = 0.f;
-          const T* kr = Ks + p * KROW;
-          const float* qh = qs + h * HD;
-#pragma unroll 4
-          for (int ee = 0; ee < HD; ee += 8) {
-            float kv[8];
-            load8s<T>(kr + ee, kv);
-            const float4 q0 = *reinterpret_cast<const float4*>(qh + ee);
-            const float4 q1 = *reinterpret_cast<const float4*>(qh + ee + 4);
-            a += kv[0] * q0.x + kv[1] * q0.y + kv[2] * q0.z + kv[3] * q0.w + kv[4] * q1.x + kv[5] * q1.y +
-                 kv[6] * q1.z + kv[7] * q1.w;
+      // logits: rounds of PPR positions x GP heads per warp, reduced over the lanes
+      {
+        constexpr int PPR = 32 / GP;                       // positions per round
+        constexpr int PPW = GP == 1 ? 32 : 16;             // positions per warp
+        constexpr int ROUNDS = PPW / PPR;
+        const int pw = warp * PPW;
+        if (pw < kChunk) {
+#pragma unroll
+          for (int r = 0; r < ROUNDS; ++r) {
+            const int pb = pw + r * PPR;
+            float v[32];
+#pragma unroll
+            for (int pi = 0; pi < PPR; ++pi) {
+              const int p = pb + pi;
+              float kd[DPL];
+              if (p < cnt) {
+                if (DPL == 4) {
+                  const uint2 u = *reinterpret_cast<const uint2*>(Ks + p * KROW + lane * 4);
+                  if (sizeof(T) == 2) {
+                    kd[0] = __uint_as_float(u.x << 16); kd[1] = __uint_as_float(u.x & 0xFFFF0000u);
+                    kd[2] = __uint_as_float(u.y << 16); kd[3] = __uint_as_float(u.y & 0xFFFF0000u);
+                  }
+                }
+                if (sizeof(T) == 4 || DPL != 4) {
+#pragma unroll
+                  for (int d = 0; d < DPL; ++d) kd[d] = to_f(Ks[p * KROW + lane * DPL + d]);
+                }
+              } else {
+#pragma unroll
+                for (int d = 0; d < DPL; ++d) kd[d] = 0.f;
+              }
+#pragma unroll
+              for (int h = 0; h < GP; ++h) {
+                float a = 0.f;
+#pragma unroll
+                for (int d = 0; d < DPL; ++d) a += qr[h][d] * kd[d];
+                v[pi * GP + h] = a;
+              }
+            }
+            // halving butterfly: lane l ends with the sum of value l
+#pragma unroll
+            for (int o = 16, nv = 16; o >= 1; o >>= 1, nv >>= 1) {
+              const bool upper = (lane & o) != 0;
+#pragma unroll
+              for (int x = 0; x < nv; ++x) {
+                const float send = upper ? v[x] : v[x + nv];
+                const float keep = upper ? v[x + nv] : v[x];
+                v[x] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+              }
+            }
+            const int p = pb + lane / GP, h = lane % GP;
+            lg[h * kChunk + p] = p < cnt ? v[0] : -INFINITY;
           }
         }
-        ps[x] = a;
       }
       sync();
-      // online softmax update, one warp per head
+      // online softmax update, one warp per head; probabilities stored by position
       for (int h = warp; h < G; h += kAttnThreads / 32) {
-        const float v0 = ps[h * kChunk + lane], v1 = ps[h * kChunk + lane + 32];
+        const float v0 = lg[h * kChunk + lane], v1 = lg[h * kChunk + lane + 32];
         const float mc = warp_max(fmaxf(v0, v1));
         const float mo = mrun_s[h];
         const float mn = fmaxf(mo, mc);
         const float e0 = (lane < cnt) ? expf(v0 - mn) : 0.f;
         const float e1 = (lane + 32 < cnt) ? expf(v1 - mn) : 0.f;
-        ps[h * kChunk + lane] = e0;
-        ps[h * kChunk + lane + 32] = e1;
+        pt[lane * GP + h] = e0;
+        pt[(lane + 32) * GP + h] = e1;
         const float sv = warp_sum(e0 + e1);
         if (lane == 0) {
           const float al = (mo == -INFINITY) ? 0.f : expf(mo - mn);
@@ -290,42 +368,73 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
           lrun_s[h] = lrun_s[h] * al + sv;
         }
       }
-      sync();
-      // P.V with rescaling of the running output
-      const int pa = half * (kChunk / SPLIT), pb = min(cnt, pa + kChunk / SPLIT);
-#pragma unroll
-      for (int h = 0; h < 8; ++h)
-        if (h < G) acc[h] *= alpha_s[h];
-      for (int p = pa; p < pb; ++p) {
-        const float v = to_f(Vs[p * HD + e]);
-#pragma unroll
-        for (int h = 0; h < 8; ++h)
-          if (h < G) acc[h] += ps[h * kChunk + p] * v;
+      for (int x = tid; x < (GP - G) * kChunk; x += kAttnThreads) {   // padded heads
+        const int h = G + x / kChunk, p = x % kChunk;
+        pt[p * GP + h] = 0.f;
+        if (p == 0) alpha_s[h] = 0.f;
       }
-      sync();   // buffer (c & 1) is refilled by the issue of chunk c + 2
-    }
-    if (SPLIT == 2) {
-      if (half == 1)
-        for (int h = 0; h < G; ++h) red[h * HD + e] = acc[h];
       sync();
-      if (half == 0)
-        for (int h = 0; h < G; ++h) acc[h] += red[h * HD + e];
-    }
-    const size_t obase = (size_t)j * nq * HD + (size_t)g * G * HD;
-    if (nsp == 1) {
-      if (half == 0)
-        for (int h = 0; h < G; ++h) store_out(out, out_lo, obase + (size_t)h * HD + e, acc[h] / lrun_s[h]);
-    } else {
-      if (half == 0) {
-        for (int h = 0; h < G; ++h) {
-          const size_t slot = ((size_t)j * nq + g * G + h) * max_spans + sp;
-          __stcg(part_acc + slot * HD + e, acc[h]);
-          if (e == 0) {
-            __stcg(part_m + slot, mrun_s[h]);
-            __stcg(part_l + slot, lrun_s[h]);
+      // P.V: channels 8*cg.. of every head over the positions of group pg
+      {
+        float al[GP];
+#pragma unroll
+        for (int h = 0; h < GP; ++h) al[h] = alpha_s[h];
+#pragma unroll
+        for (int h = 0; h < GP; ++h)
+#pragma unroll
+          for (int k = 0; k < 8; ++k) acc[h][k] *= al[h];
+#pragma unroll
+        for (int u = 0; u < PPG; ++u) {
+          const int p = pg * PPG + u;
+          if (p < cnt) {
+            float v8[8];
+            load8s<T>(Vs + p * HD + cg * 8, v8);
+            float pv[GP];
+            if (GP >= 4) {
+#pragma unroll
+              for (int h4 = 0; h4 < GP; h4 += 4) {
+                const float4 t4 = *reinterpret_cast<const float4*>(pt + p * GP + h4);
+                pv[h4] = t4.x; pv[h4 + 1] = t4.y; pv[h4 + 2] = t4.z; pv[h4 + 3] = t4.w;
+              }
+            } else {
+#pragma unroll
+              for (int h = 0; h < GP; ++h) pv[h] = pt[p * GP + h];
+            }
+#pragma unroll
+            for (int h = 0; h < GP; ++h)
+#pragma unroll
+              for (int k = 0; k < 8; ++k) acc[h][k] += pv[h] * v8[k];
           }
         }
       }
+      sync();   // buffer (c & 1) is refilled by the issue of chunk c + 2
+    }
+    // sum the position groups (the K buffers are free now)
+#pragma unroll
+    for (int h = 0; h < GP; ++h) {
+      float4* r = reinterpret_cast<float4*>(red + ((size_t)pg * GP + h) * HD + cg * 8);
+      r[0] = make_float4(acc[h][0], acc[h][1], acc[h][2], acc[h][3]);
+      r[1] = make_float4(acc[h][4], acc[h][5], acc[h][6], acc[h][7]);
+    }
+    sync();
+    const size_t obase = (size_t)j * nq * HD + (size_t)g * G * HD;
+    for (int x = tid; x < G * HD; x += kAttnThreads) {
+      const int h = x / HD, e = x - h * HD;
+      float o = 0.f;
+#pragma unroll
+      for (int q2 = 0; q2 < NPG; ++q2) o += red[((size_t)q2 * GP + h) * HD + e];
+      if (nsp == 1) {
+        store_out(out, out_lo, obase + x, o / lrun_s[h]);
+      } else {
+        const size_t slot = ((size_t)j * nq + g * G + h) * max_spans + sp;
+        __stcg(part_acc + slot * HD + e, o);
+        if (e == 0) {
+          __stcg(part_m + slot, mrun_s[h]);
+          __stcg(part_l + slot, lrun_s[h]);
+        }
+      }
+    }
+    if (nsp > 1) {
       sync();
       if (tid == 0) {
         __threadfence();
@@ -336,8 +445,9 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
       }
       sync();
       if (*last_s_p) {
-        // merge in span order: per head the weights exp(m_s - M), then every
-        // output channel as independent loads over the spans
+        // merge in span order: per head the weights exp(m_s - M), then four
+        // consecutive channels per thread with the partials of sixteen spans
+        // loaded together and accumulated in span order
         for (int h = warp; h < G; h += kAttnThreads / 32) {
           const size_t base = ((size_t)j * nq + g * G + h) * max_spans;
           float mloc = -INFINITY;
@@ -353,20 +463,18 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
           if (lane == 0) lrun_s[h] = lsum;
         }
         sync();
-        // four consecutive channels per thread; the partials of eight spans
-        // are loaded together, then accumulated in span order
         for (int x4 = tid; x4 < G * HD / 4; x4 += kAttnThreads) {
           const int h = (x4 * 4) / HD, ee = x4 * 4 - h * HD;
           const float* pa0 = part_acc + ((size_t)j * nq + g * G + h) * max_spans * HD + ee;
           const float* wh = wch + h * max_spans;
           float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-          for (int c0 = 0; c0 < nsp; c0 += 8) {
-            float4 t[8];
+          for (int c0 = 0; c0 < nsp; c0 += 16) {
+            float4 t[16];
 #pragma unroll
-            for (int k = 0; k < 8; ++k)
+            for (int k = 0; k < 16; ++k)
               if (c0 + k < nsp) t[k] = __ldcg(reinterpret_cast<const float4*>(pa0 + (size_t)(c0 + k) * HD));
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
+            for (int k = 0; k < 16; ++k) {
               if (c0 + k < nsp) {
                 const float w = wh[c0 + k];
                 a.x += t[k].x * w;

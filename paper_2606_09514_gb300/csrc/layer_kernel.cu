@@ -57,6 +57,7 @@ struct LkParams {
   unsigned* bar;         // grid barrier: [0] arrivals, [1] generation
   TcParams tp[4];        // epilogue parameters of each GEMM
   AttnArgs<bf16> attn;
+  int attn_gp;           // padded query heads per KV head (attention template)
   int32_t* status;
 };
 
@@ -332,7 +333,13 @@ __global__ void __launch_bounds__(kLkThreads, 1)
                                               &last_flag);
     if (ok) ok = lk_grid_sync(p.bar, gen, &abort_flag, &passed, &ok_s, p.status);                  // B2
     if (ok) {
-      attn_run<bf16, 128>(p.attn, t, blockIdx.x, gridDim.x, smem + p.attn_off, sc, SyncEpilogueWarps{}, false);
+      uint8_t* as = smem + p.attn_off;
+      switch (p.attn_gp) {
+        case 1: attn_run<bf16, 128, 1>(p.attn, t, blockIdx.x, gridDim.x, as, sc, SyncEpilogueWarps{}, false); break;
+        case 2: attn_run<bf16, 128, 2>(p.attn, t, blockIdx.x, gridDim.x, as, sc, SyncEpilogueWarps{}, false); break;
+        case 4: attn_run<bf16, 128, 4>(p.attn, t, blockIdx.x, gridDim.x, as, sc, SyncEpilogueWarps{}, false); break;
+        default: attn_run<bf16, 128, 8>(p.attn, t, blockIdx.x, gridDim.x, as, sc, SyncEpilogueWarps{}, false);
+      }
       ok = lk_grid_sync(p.bar, gen, &abort_flag, &passed, &ok_s, p.status);                        // B3
     }
     if (ok) ok = lk_epilogue<EPI_RESID, SPLIT>(p, 1, m, tmem_base, tfull_bar, tempty_bar, acc, acc_ph, &abort_flag,
@@ -434,6 +441,7 @@ bool launch_layer_kernel(const Ctx& c, const buddy_kv_state& kv, int l, RowSel s
                           (const bf16*)kv.k_cache[l], (const bf16*)kv.v_cache[l], c.attn_max_chunks, c.attn_m,
                           c.attn_l, c.attn_acc, c.attn_ctr, (bf16*)c.attn_out, split ? (bf16*)c.attn_lo : nullptr,
                           c.status};
+  p.attn_gp = attn_group_pad(G);
   p.status = c.status;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(c.num_sms);
