@@ -30,9 +30,10 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "budget-routed decode tokens/s at 1 GB300 per budget; % of HBM/tensor roofline"
-# ncu dram bytes per launch of the dominant kernel, from the committed profile
-# summary of the current kernel (None until captured for this kernel version)
-NCU_TRAFFIC_PER_LAUNCH = {}
+# ncu dram bytes (read + write) per launch of the dominant kernel, from the
+# committed ncu summary of the gate/up GEMM (3-layer model with the same layer
+# shapes as the 32-layer bench workload); absent for kernels not captured
+NCU_TRAFFIC_PER_LAUNCH = {"gemm_gate_up": 237988608}
 
 
 def _peaks():
