@@ -122,6 +122,14 @@ def test_budget_one_and_batch_one():
     run_parity(w, steps=3)
 
 
+def test_decode_parity_three_rows_graph_prior():
+    """Three rows (a single 16-row MMA tile, most of it padding) with bias,
+    RoPE partners, ragged contexts, the prior and the graph."""
+    w = C.scaled(C.T_QWEN, ctx=[0, 129, 700], k=[1, 5, 3], name="t-qwen-b3")
+    worst, _ = run_parity(w, steps=3, use_graph=True, prior=True)
+    assert worst < 2e-2
+
+
 def test_graph_replay_equals_direct_launches():
     w = C.T_GQA
     outs = []
