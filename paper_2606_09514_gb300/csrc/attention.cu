@@ -28,7 +28,7 @@ template <typename T, int HD, int GP>
 __global__ void __launch_bounds__(kAttnThreads) attn_kernel(AttnArgs<T> A) {
   extern __shared__ __align__(16) uint8_t smraw[];
   __shared__ float sc[32];
-  attn_run<T, HD, GP>(A, threadIdx.x, blockIdx.x, gridDim.x, smraw, sc, SyncCta{}, true);
+  attn_run<T, HD, GP, kAttnThreads>(A, threadIdx.x, blockIdx.x, gridDim.x, smraw, sc, SyncCta{}, true);
 }
 
 template <typename T, int HD, int GP>

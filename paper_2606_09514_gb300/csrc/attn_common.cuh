@@ -11,7 +11,7 @@
 namespace buddy {
 
 constexpr int kChunk = 64;
-constexpr int kAttnThreads = 128;
+constexpr int kAttnThreads = 256;   // the attention kernel's CTA (the per-layer kernel uses 128)
 constexpr int kMaxSpan = 1024;
 
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
@@ -101,7 +101,7 @@ inline size_t attn_smem_bytes(size_t fixed, int G, int hd, int max_spans, int ma
 inline int attn_group_pad(int G) { return G <= 1 ? 1 : (G <= 2 ? 2 : (G <= 4 ? 4 : 8)); }
 
 // Processes this CTA's share (items cta, cta + ncta, ...) of one layer's
-// attention with kAttnThreads threads numbered tid; `sync` synchronises them;
+// attention with NT threads numbered tid; `sync` synchronises them;
 // `sc` points to 32 floats of shared scratch.  With `pdl` the copies that do
 // not depend on the preceding kernel start before waiting on it.  GP >= G is
 // the padded number of query heads per KV head.
@@ -116,7 +116,7 @@ inline int attn_group_pad(int G) { return G <= 1 ? 1 : (G <= 2 ? 2 : (G <= 4 ? 4
 //           positions of group t / (HD/8); its partial sums stay in registers
 //           across the chunks of the span (rescaled by the online-softmax
 //           factor) and the groups are summed once at the end of the span.
-template <typename T, int HD, int GP, typename Sync>
+template <typename T, int HD, int GP, int NT, typename Sync>
 __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta, int ncta, uint8_t* smem,
                                          float* sc, Sync sync, bool pdl) {
   static_assert(GP == 1 || GP == 2 || GP == 4 || GP == 8, "GP");
@@ -154,7 +154,8 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
   constexpr int V16 = HD * (int)sizeof(T) / 16;  // 16-byte pieces per row
   constexpr int E16 = 16 / sizeof(T);            // elements per piece
   constexpr int CH = HD / 8;                     // P.V channel groups of 8
-  constexpr int NPG = kAttnThreads / CH;         // P.V position groups
+  constexpr int NPG = NT / CH;                   // P.V position groups
+  constexpr int NW = NT / 32;                    // warps
   constexpr int PPG = kChunk / NPG;              // positions per group and chunk
   const int G = nq / nkv;
   T* Kb0 = reinterpret_cast<T*>(smem);                          // 2 x [kChunk][KROW]
@@ -168,7 +169,7 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
       (reinterpret_cast<uintptr_t>(pref + m + 1) + 7) & ~uintptr_t(7));
   int* rnp = reinterpret_cast<int*>(rbase + m);                 // [m] positions (len + 1)
   int* rhs = rnp + m;                                           // [m] head stride (cap * HD)
-  float* red = reinterpret_cast<float*>(Kb0);                   // [NPG][GP][HD], after the last chunk
+  float* red = reinterpret_cast<float*>(Kb0);                   // [NPG][HR][HD], after the last chunk
   float* alpha_s = sc;        // [8]
   float* mrun_s = sc + 8;     // [8]
   float* lrun_s = sc + 16;    // [8]
@@ -244,7 +245,7 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
       const int p0 = s0 + c * kChunk, cnt = min(kChunk, s1 - p0);
       T* Kd = Kb0 + (c & 1) * kChunk * KROW;
       T* Vd = Vb0 + (c & 1) * kChunk * HD;
-      for (int x = tid; x < cnt * V16; x += kAttnThreads) {
+      for (int x = tid; x < cnt * V16; x += NT) {
         const int p = x / V16, s = x - p * V16;
         cp_async16(Kd + p * KROW + s * E16, Kbase + (size_t)(p0 + p) * HD + s * E16);
         cp_async16(Vd + p * HD + s * E16, Vbase + (size_t)(p0 + p) * HD + s * E16);
@@ -264,7 +265,7 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
       issue(0);
     }
     const float* qj = q + (size_t)j * nq * HD + (size_t)g * G * HD;
-    for (int x = tid; x < GP * HD; x += kAttnThreads) qs[x] = x < G * HD ? qj[x] * scale : 0.f;
+    for (int x = tid; x < GP * HD; x += NT) qs[x] = x < G * HD ? qj[x] * scale : 0.f;
     sync();
     // this lane's query dims for the logits
     constexpr int DPL = HD / 32;
@@ -296,8 +297,8 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
       const T* Vs = Vb0 + (c & 1) * kChunk * HD;
       // logits: rounds of PPR positions x GP heads per warp, reduced over the lanes
       {
-        constexpr int PPR = 32 / GP;                       // positions per round
-        constexpr int PPW = GP == 1 ? 32 : 16;             // positions per warp
+        constexpr int PPR = 32 / GP;                                    // positions per round
+        constexpr int PPW = kChunk / NW > PPR ? kChunk / NW : PPR;      // positions per warp
         constexpr int ROUNDS = PPW / PPR;
         const int pw = warp * PPW;
         if (pw < kChunk) {
@@ -351,7 +352,7 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
       }
       sync();
       // online softmax update, one warp per head; probabilities stored by position
-      for (int h = warp; h < G; h += kAttnThreads / 32) {
+      for (int h = warp; h < G; h += NW) {
         const float v0 = lg[h * kChunk + lane], v1 = lg[h * kChunk + lane + 32];
         const float mc = warp_max(fmaxf(v0, v1));
         const float mo = mrun_s[h];
@@ -368,7 +369,7 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
           lrun_s[h] = lrun_s[h] * al + sv;
         }
       }
-      for (int x = tid; x < (GP - G) * kChunk; x += kAttnThreads) {   // padded heads
+      for (int x = tid; x < (GP - G) * kChunk; x += NT) {   // padded heads
         const int h = G + x / kChunk, p = x % kChunk;
         pt[p * GP + h] = 0.f;
         if (p == 0) alpha_s[h] = 0.f;
@@ -409,28 +410,39 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
       }
       sync();   // buffer (c & 1) is refilled by the issue of chunk c + 2
     }
-    // sum the position groups (the K buffers are free now)
-#pragma unroll
-    for (int h = 0; h < GP; ++h) {
-      float4* r = reinterpret_cast<float4*>(red + ((size_t)pg * GP + h) * HD + cg * 8);
-      r[0] = make_float4(acc[h][0], acc[h][1], acc[h][2], acc[h][3]);
-      r[1] = make_float4(acc[h][4], acc[h][5], acc[h][6], acc[h][7]);
-    }
-    sync();
+    // sum the position groups (the K and V buffers are free now), in passes
+    // of HR heads when [NPG][GP][HD] floats do not fit there
+    constexpr size_t kKVBytes = 2 * (size_t)kChunk * KROW * sizeof(T) + 2 * (size_t)kChunk * HD * sizeof(T);
+    constexpr int HR = (size_t)NPG * GP * HD * 4 <= kKVBytes
+                           ? GP
+                           : ((size_t)NPG * (GP / 2) * HD * 4 <= kKVBytes ? GP / 2 : (GP >= 4 ? GP / 4 : 1));
+    static_assert((size_t)NPG * HR * HD * 4 <= kKVBytes, "attention reduction buffer");
     const size_t obase = (size_t)j * nq * HD + (size_t)g * G * HD;
-    for (int x = tid; x < G * HD; x += kAttnThreads) {
-      const int h = x / HD, e = x - h * HD;
-      float o = 0.f;
 #pragma unroll
-      for (int q2 = 0; q2 < NPG; ++q2) o += red[((size_t)q2 * GP + h) * HD + e];
-      if (nsp == 1) {
-        store_out(out, out_lo, obase + x, o / lrun_s[h]);
-      } else {
-        const size_t slot = ((size_t)j * nq + g * G + h) * max_spans + sp;
-        __stcg(part_acc + slot * HD + e, o);
-        if (e == 0) {
-          __stcg(part_m + slot, mrun_s[h]);
-          __stcg(part_l + slot, lrun_s[h]);
+    for (int h0 = 0; h0 < GP; h0 += HR) {
+      if (h0 > 0) sync();   // the previous pass has read the buffer
+#pragma unroll
+      for (int hh = 0; hh < HR; ++hh) {
+        float4* r = reinterpret_cast<float4*>(red + ((size_t)pg * HR + hh) * HD + cg * 8);
+        r[0] = make_float4(acc[h0 + hh][0], acc[h0 + hh][1], acc[h0 + hh][2], acc[h0 + hh][3]);
+        r[1] = make_float4(acc[h0 + hh][4], acc[h0 + hh][5], acc[h0 + hh][6], acc[h0 + hh][7]);
+      }
+      sync();
+      for (int x = tid; x < HR * HD; x += NT) {
+        const int hh = x / HD, e = x - hh * HD, h = h0 + hh;
+        if (h >= G) continue;
+        float o = 0.f;
+#pragma unroll
+        for (int q2 = 0; q2 < NPG; ++q2) o += red[((size_t)q2 * HR + hh) * HD + e];
+        if (nsp == 1) {
+          store_out(out, out_lo, obase + (size_t)h * HD + e, o / lrun_s[h]);
+        } else {
+          const size_t slot = ((size_t)j * nq + g * G + h) * max_spans + sp;
+          __stcg(part_acc + slot * HD + e, o);
+          if (e == 0) {
+            __stcg(part_m + slot, mrun_s[h]);
+            __stcg(part_l + slot, lrun_s[h]);
+          }
         }
       }
     }
@@ -448,7 +460,7 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
         // merge in span order: per head the weights exp(m_s - M), then four
         // consecutive channels per thread with the partials of sixteen spans
         // loaded together and accumulated in span order
-        for (int h = warp; h < G; h += kAttnThreads / 32) {
+        for (int h = warp; h < G; h += NW) {
           const size_t base = ((size_t)j * nq + g * G + h) * max_spans;
           float mloc = -INFINITY;
           for (int cc = lane; cc < nsp; cc += 32) mloc = fmaxf(mloc, __ldcg(part_m + base + cc));
@@ -463,7 +475,7 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
           if (lane == 0) lrun_s[h] = lsum;
         }
         sync();
-        for (int x4 = tid; x4 < G * HD / 4; x4 += kAttnThreads) {
+        for (int x4 = tid; x4 < G * HD / 4; x4 += NT) {
           const int h = (x4 * 4) / HD, ee = x4 * 4 - h * HD;
           const float* pa0 = part_acc + ((size_t)j * nq + g * G + h) * max_spans * HD + ee;
           const float* wh = wch + h * max_spans;

@@ -335,10 +335,10 @@ __global__ void __launch_bounds__(kLkThreads, 1)
     if (ok) {
       uint8_t* as = smem + p.attn_off;
       switch (p.attn_gp) {
-        case 1: attn_run<bf16, 128, 1>(p.attn, t, blockIdx.x, gridDim.x, as, sc, SyncEpilogueWarps{}, false); break;
-        case 2: attn_run<bf16, 128, 2>(p.attn, t, blockIdx.x, gridDim.x, as, sc, SyncEpilogueWarps{}, false); break;
-        case 4: attn_run<bf16, 128, 4>(p.attn, t, blockIdx.x, gridDim.x, as, sc, SyncEpilogueWarps{}, false); break;
-        default: attn_run<bf16, 128, 8>(p.attn, t, blockIdx.x, gridDim.x, as, sc, SyncEpilogueWarps{}, false);
+        case 1: attn_run<bf16, 128, 1, 128>(p.attn, t, blockIdx.x, gridDim.x, as, sc, SyncEpilogueWarps{}, false); break;
+        case 2: attn_run<bf16, 128, 2, 128>(p.attn, t, blockIdx.x, gridDim.x, as, sc, SyncEpilogueWarps{}, false); break;
+        case 4: attn_run<bf16, 128, 4, 128>(p.attn, t, blockIdx.x, gridDim.x, as, sc, SyncEpilogueWarps{}, false); break;
+        default: attn_run<bf16, 128, 8, 128>(p.attn, t, blockIdx.x, gridDim.x, as, sc, SyncEpilogueWarps{}, false);
       }
       ok = lk_grid_sync(p.bar, gen, &abort_flag, &passed, &ok_s, p.status);                        // B3
     }
