@@ -85,16 +85,17 @@ struct AttnArgs {
 
 // Dynamic shared memory used by attn_run (bytes): double-buffered K (rows
 // padded by 16 bytes) and V chunks, the scaled queries, the logits, the
-// probabilities by position, the span-merge weights, the row prefix and the
-// rows' cache offsets, positions and head strides.
+// probabilities by position, the row prefix and the rows' cache offsets,
+// positions and head strides.
 template <typename T, int HD>
 __host__ __device__ constexpr size_t attn_smem_fixed() {
   return 2 * (size_t)kChunk * (HD + 16 / sizeof(T)) * sizeof(T) + 2 * (size_t)kChunk * HD * sizeof(T);
 }
 inline size_t attn_smem_bytes(size_t fixed, int G, int hd, int max_spans, int max_rows) {
   const int gp = G <= 1 ? 1 : (G <= 2 ? 2 : (G <= 4 ? 4 : 8));
-  return fixed + (size_t)gp * hd * 4 + 2 * (size_t)gp * kChunk * 4 + (size_t)gp * max_spans * 4 +
-         (size_t)(max_rows + 1) * 4 + 8 + (size_t)max_rows * 16;
+  (void)max_spans;
+  return fixed + (size_t)gp * hd * 4 + 2 * (size_t)gp * kChunk * 4 + (size_t)(max_rows + 1) * 4 + 8 +
+         (size_t)max_rows * 16;
 }
 
 // Query heads per KV head rounded up to 1, 2, 4 or 8 (the work-loop template).
@@ -163,8 +164,7 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
   float* qs = reinterpret_cast<float*>(Vb0 + 2 * kChunk * HD);  // [GP][HD]
   float* lg = qs + GP * HD;                                     // [GP][kChunk] logits
   float* pt = lg + GP * kChunk;                                 // [kChunk][GP] probabilities
-  float* wch = pt + GP * kChunk;                                // [GP][max_spans] merge weights
-  int* pref = reinterpret_cast<int*>(wch + GP * max_spans);     // [m + 1] span prefix over rows
+  int* pref = reinterpret_cast<int*>(pt + GP * kChunk);         // [m + 1] span prefix over rows
   int64_t* rbase = reinterpret_cast<int64_t*>(                  // [m] cache offset of each row
       (reinterpret_cast<uintptr_t>(pref + m + 1) + 7) & ~uintptr_t(7));
   int* rnp = reinterpret_cast<int*>(rbase + m);                 // [m] positions (len + 1)
@@ -457,51 +457,67 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
       }
       sync();
       if (*last_s_p) {
-        // merge in span order: per head the weights exp(m_s - M), then four
-        // consecutive channels per thread with the partials of sixteen spans
-        // loaded together and accumulated in span order
-        for (int h = warp; h < G; h += NW) {
-          const size_t base = ((size_t)j * nq + g * G + h) * max_spans;
-          float mloc = -INFINITY;
-          for (int cc = lane; cc < nsp; cc += 32) mloc = fmaxf(mloc, __ldcg(part_m + base + cc));
-          const float M = warp_max(mloc);
-          float lsum = 0.f;
-          for (int cc = lane; cc < nsp; cc += 32) {
-            const float w = expf(__ldcg(part_m + base + cc) - M);
-            wch[h * max_spans + cc] = w;
-            lsum += __ldcg(part_l + base + cc) * w;
-          }
-          lsum = warp_sum(lsum);
-          if (lane == 0) lrun_s[h] = lsum;
-        }
-        sync();
-        for (int x4 = tid; x4 < G * HD / 4; x4 += NT) {
-          const int h = (x4 * 4) / HD, ee = x4 * 4 - h * HD;
-          const float* pa0 = part_acc + ((size_t)j * nq + g * G + h) * max_spans * HD + ee;
-          const float* wh = wch + h * max_spans;
+        // merge: the tpo adjacent threads of an output (four consecutive
+        // channels of one head) take spans sub, sub + tpo, ... with a running
+        // rescaled sum (running max M, sum L, output a), loading sixteen of
+        // their spans' partials at a time; the tpo results are then combined
+        // by a lane butterfly (every thread ends with the same values)
+        const int n4 = G * HD / 4;
+        int tpo = 1;
+        while (tpo < 8 && tpo * 2 * n4 <= NT) tpo *= 2;
+        const int x4 = tid / tpo, sub = tid % tpo;
+        if (tid < ((n4 * tpo + 31) & ~31)) {   // whole warps take part in the butterfly
+          const bool act = x4 < n4;
+          const int h = act ? (x4 * 4) / HD : 0, ee = act ? x4 * 4 - h * HD : 0;
+          const size_t hb = ((size_t)j * nq + g * G + h) * max_spans;
+          float M = -INFINITY, L = 0.f;
           float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-          for (int c0 = 0; c0 < nsp; c0 += 16) {
+          for (int c0 = sub; act && c0 < nsp; c0 += 16 * tpo) {
             float4 t[16];
-#pragma unroll
-            for (int k = 0; k < 16; ++k)
-              if (c0 + k < nsp) t[k] = __ldcg(reinterpret_cast<const float4*>(pa0 + (size_t)(c0 + k) * HD));
+            float ms[16], ls[16];
 #pragma unroll
             for (int k = 0; k < 16; ++k) {
-              if (c0 + k < nsp) {
-                const float w = wh[c0 + k];
-                a.x += t[k].x * w;
-                a.y += t[k].y * w;
-                a.z += t[k].z * w;
-                a.w += t[k].w * w;
+              const int cc = c0 + k * tpo;
+              if (cc < nsp) {
+                t[k] = __ldcg(reinterpret_cast<const float4*>(part_acc + (hb + cc) * HD + ee));
+                ms[k] = __ldcg(part_m + hb + cc);
+                ls[k] = __ldcg(part_l + hb + cc);
+              }
+            }
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+              if (c0 + k * tpo < nsp) {
+                const float mn = fmaxf(M, ms[k]);
+                const float fo = expf(M - mn), fn = expf(ms[k] - mn);
+                a.x = a.x * fo + t[k].x * fn;
+                a.y = a.y * fo + t[k].y * fn;
+                a.z = a.z * fo + t[k].z * fn;
+                a.w = a.w * fo + t[k].w * fn;
+                L = L * fo + ls[k] * fn;
+                M = mn;
               }
             }
           }
-          const float l = lrun_s[h];
-          const size_t o = obase + (size_t)h * HD + ee;
-          store_out(out, out_lo, o + 0, a.x / l);
-          store_out(out, out_lo, o + 1, a.y / l);
-          store_out(out, out_lo, o + 2, a.z / l);
-          store_out(out, out_lo, o + 3, a.w / l);
+          for (int o = 1; o < tpo; o <<= 1) {
+            const float M2 = __shfl_xor_sync(0xffffffffu, M, o), L2 = __shfl_xor_sync(0xffffffffu, L, o);
+            const float ax = __shfl_xor_sync(0xffffffffu, a.x, o), ay = __shfl_xor_sync(0xffffffffu, a.y, o);
+            const float az = __shfl_xor_sync(0xffffffffu, a.z, o), aw = __shfl_xor_sync(0xffffffffu, a.w, o);
+            const float mn = fmaxf(M, M2);
+            const float f1 = M == -INFINITY ? 0.f : expf(M - mn), f2 = M2 == -INFINITY ? 0.f : expf(M2 - mn);
+            a.x = a.x * f1 + ax * f2;
+            a.y = a.y * f1 + ay * f2;
+            a.z = a.z * f1 + az * f2;
+            a.w = a.w * f1 + aw * f2;
+            L = L * f1 + L2 * f2;
+            M = mn;
+          }
+          if (act && sub == 0) {
+            const size_t o = obase + (size_t)h * HD + ee;
+            store_out(out, out_lo, o + 0, a.x / L);
+            store_out(out, out_lo, o + 1, a.y / L);
+            store_out(out, out_lo, o + 2, a.z / L);
+            store_out(out, out_lo, o + 3, a.w / L);
+          }
         }
       }
     }
