@@ -326,7 +326,13 @@ def run_ours(args, ws, rank, local):
     step_s = ms_max / 1e3 / K
     route_frac = (prof["route"][0] + prof["compact"][0]) / max(prof_ms_total, 1e-9)
     launches_per_step = sum(v[1] for v in prof.values()) / prof_steps
-    graph_extra = (s.n_layers - 2) if not args.no_graph else 0   # conditional-setting kernels
+    # the timed steps launch every middle layer (a layer no row selected exits
+    # at once); the profiled steps launch only the selected ones
+    per_layer = ("rmsnorm", "gemm_qkv", "qkv_finalize", "attention", "gemm_o", "gemm_gate_up", "gemm_down",
+                 "layer")
+    exec_layers = (prof.get("gemm_gate_up", (0, 0))[1] + prof.get("layer", (0, 0))[1]) / prof_steps
+    per_layer_kernels = sum(prof.get(k, (0, 0))[1] for k in per_layer) / max(exec_layers * prof_steps, 1)
+    graph_extra = max(s.n_layers - exec_layers, 0) * per_layer_kernels
     out = {
         "metric": METRIC, "value": round(value, 2), "unit": "tokens/s", "n_gpus": ws, "steps": K,
         "warmup": W, "ms_per_step": round(ms_max / K, 4), "higher_is_better": True, "scaling": "weak",

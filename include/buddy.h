@@ -213,10 +213,10 @@ BUDDY_API int buddy_decode_step_host(buddy_ctx* ctx, const buddy_kv_state* kv, i
                            uint8_t* mask_host, void* stream);
 
 /* Execution options.  use_graph != 0: buddy_decode_step replays a CUDA graph
- * captured per (batch, kv state, stream) on first use, with a device-set
- * conditional node per layer so that layers no sequence selected cost no
- * kernel launches.  The graph bakes in the pointers of that call; a call with
- * other pointers re-captures. */
+ * of the step's launches, captured per (batch, kv state, stream) on first use;
+ * the kernels of a layer that no sequence selected exit as soon as they start.
+ * The graph bakes in the pointers of that call; a call with other pointers
+ * re-captures. */
 BUDDY_API int buddy_set_options(buddy_ctx* ctx, int32_t use_graph);
 
 /* Kernel classes reported by the profiler. */

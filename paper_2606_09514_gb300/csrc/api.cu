@@ -1,6 +1,6 @@
 // C-ABI of libbuddy: argument validation, scratch management, and the
 // orchestration of one budget-routed decode step (direct launches or a CUDA
-// graph whose middle layers sit behind device-set conditional nodes).
+// graph of the same launches; layers no sequence selected exit at once).
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -20,7 +20,6 @@ using namespace buddy;
 struct buddy_ctx {
   Ctx c;
   cudaStream_t cap_stream = nullptr;   // graph capture (the legacy stream cannot be captured)
-  cudaStream_t body_stream = nullptr;  // capture of conditional bodies
 };
 
 #define CK(x)                                                     \
@@ -60,7 +59,6 @@ static void free_ctx(buddy_ctx* x) {
   for (void* p : ptrs)
     if (p) cudaFree(p);
   if (x->cap_stream) cudaStreamDestroy(x->cap_stream);
-  if (x->body_stream) cudaStreamDestroy(x->body_stream);
   delete x;
 }
 
@@ -146,9 +144,7 @@ extern "C" int buddy_create(const buddy_config* cfg, buddy_ctx** out) {
   if ((e = cudaMemset(c.status, 0, 4 * sizeof(int32_t))) != cudaSuccess ||
       (e = cudaMemset(c.attn_ctr, 0, B * c.nkv * sizeof(int32_t))) != cudaSuccess)
     return fail(e);
-  if ((e = cudaStreamCreateWithFlags(&x->cap_stream, cudaStreamNonBlocking)) != cudaSuccess ||
-      (e = cudaStreamCreateWithFlags(&x->body_stream, cudaStreamNonBlocking)) != cudaSuccess)
-    return fail(e);
+  if ((e = cudaStreamCreateWithFlags(&x->cap_stream, cudaStreamNonBlocking)) != cudaSuccess) return fail(e);
   launch_rope_table(c.rope_cos, c.rope_sin, c.max_pos, c.hd, (double)g.rope_theta, x->cap_stream);
   if ((e = cudaGetLastError()) != cudaSuccess || (e = cudaStreamSynchronize(x->cap_stream)) != cudaSuccess)
     return fail(e);
@@ -378,9 +374,9 @@ struct StepIO {
   float* scores_out;
 };
 
-// Enqueues the whole step.  When `body_stream` is non-null the caller is
-// capturing `s` into a graph: each middle layer becomes a conditional node
-// whose body runs iff count[l] > 0.
+// Enqueues the whole step on `s` (which the caller may be capturing into a
+// graph).  With profiling, the host reads the layer counts and launches only
+// the layers some sequence selected.
 static int enqueue_step(buddy_ctx* x, const buddy_kv_state& kv, const StepIO& io, cudaStream_t s,
                         bool capture) {
   Ctx& c = x->c;
@@ -406,42 +402,14 @@ static int enqueue_step(buddy_ctx* x, const buddy_kv_state& kv, const StepIO& io
     CK(cudaMemcpyAsync(hcount, c.count, sizeof(int32_t) * c.L, cudaMemcpyDeviceToHost, s));
     CK(cudaStreamSynchronize(s));
   }
-  cudaGraphConditionalHandle handles[kMaxLayers];
-  if (capture) {
-    // one handle per middle layer, all set by a single kernel after compaction
-    cudaGraph_t g = nullptr;
-    cudaStreamCaptureStatus st;
-    CK(cudaStreamGetCaptureInfo(s, &st, nullptr, &g, nullptr, nullptr, nullptr));
-    for (int l = 1; l < c.L - 1; ++l)
-      CK(cudaGraphConditionalHandleCreate(&handles[l - 1], g, 0, cudaGraphCondAssignDefault));
-    launch_set_conditionals(handles, c.L - 2, c.count, c.status, s);
-  }
+  // Every middle layer is enqueued; a layer that no sequence selected costs one
+  // early exit per kernel (its row count, written by the compaction kernel, is
+  // read before any setup).  Graph conditional nodes would skip those launches
+  // but cut the programmatic-dependent-launch overlap at every executed layer,
+  // which costs more at the budgets of interest.
   for (int l = 1; l < c.L - 1; ++l) {
     const RowSel sel{c.rows + (size_t)l * B, c.count + l, B};
-    if (!capture) {
-      if (!prof || hcount[l] > 0) enqueue_layer(c, kv, l, sel, io.h_out, io.h_out, s, prof);
-      continue;
-    }
-    cudaGraph_t g = nullptr;
-    cudaStreamCaptureStatus st;
-    const cudaGraphNode_t* deps = nullptr;
-    const cudaGraphEdgeData* edata = nullptr;
-    size_t ndeps = 0;
-    CK(cudaStreamGetCaptureInfo(s, &st, nullptr, &g, &deps, &edata, &ndeps));
-    cudaGraphNodeParams p{};
-    p.type = cudaGraphNodeTypeConditional;
-    p.conditional.handle = handles[l - 1];
-    p.conditional.type = cudaGraphCondTypeIf;
-    p.conditional.size = 1;
-    cudaGraphNode_t node;
-    CK(cudaGraphAddNode(&node, g, deps, edata, ndeps, &p));
-    cudaGraph_t body = p.conditional.phGraph_out[0];
-    CK(cudaStreamUpdateCaptureDependencies(s, &node, nullptr, 1, cudaStreamSetCaptureDependencies));
-    CK(cudaStreamBeginCaptureToGraph(x->body_stream, body, nullptr, nullptr, 0,
-                                     cudaStreamCaptureModeRelaxed));
-    enqueue_layer(c, kv, l, sel, io.h_out, io.h_out, x->body_stream, false);
-    cudaGraph_t done = nullptr;
-    CK(cudaStreamEndCapture(x->body_stream, &done));
+    if (!prof || hcount[l] > 0) enqueue_layer(c, kv, l, sel, io.h_out, io.h_out, s, prof);
   }
   enqueue_layer(c, kv, c.L - 1, all, io.h_out, io.h_out, s, prof);
   {

@@ -45,6 +45,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
 
+  // A layer that no row selected leaves before any setup.  Its row count was
+  // written by the compaction kernel, which completed before the preceding
+  // kernel of the step let this one launch (every kernel of the step waits on
+  // its predecessor before allowing its dependents to start), so it may be read
+  // before the wait.  The wait itself still happens, so that the completion of
+  // this kernel implies the completion of everything enqueued before it.
+  if (p.count && *reinterpret_cast<const volatile int32_t*>(p.count) <= 0) {
+    pdl_wait();
+    pdl_trigger();
+    return;
+  }
+
   if (threadIdx.x == 0) {
     for (int s = 0; s < p.stages; ++s) {
       ptx::mbar_init(&full_bar[s], 1);

@@ -107,9 +107,6 @@ void launch_kv_append(const Ctx& c, const buddy_kv_state& kv, int layer, int n_s
                       cudaStream_t s);
 void launch_pool_refresh(const Ctx& c, const buddy_kv_state& kv, int n_seq, const int32_t* seq_ids,
                          int n_new, cudaStream_t s);
-void launch_set_conditionals(const cudaGraphConditionalHandle* h, int n, const int32_t* count,
-                             const int32_t* status, cudaStream_t s);
-
 // GEMMs (gemm_simt.cu, gemm_tc.cu)
 void launch_gemm_simt(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s);
 bool gemm_tc_supported(const Ctx& c);

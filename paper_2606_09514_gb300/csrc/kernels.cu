@@ -512,26 +512,4 @@ void launch_pool_refresh(const Ctx& c, const buddy_kv_state& kv, int n_seq, cons
                                                  c.status);
 }
 
-// ---------------------------------------------------------------------------
-// Graph conditionals: layer l's body runs iff some sequence selected it.  One
-// thread per middle layer sets that layer's handle.
-// ---------------------------------------------------------------------------
-struct CondHandles {
-  cudaGraphConditionalHandle h[kMaxLayers];
-};
-
-__global__ void set_conditionals_kernel(CondHandles hs, int n, const int32_t* count, const int32_t* status) {
-  const int t = threadIdx.x;
-  if (t >= n) return;
-  const bool run = !call_aborted(status) && count[t + 1] > 0;
-  cudaGraphSetConditional(hs.h[t], run ? 1u : 0u);
-}
-
-void launch_set_conditionals(const cudaGraphConditionalHandle* h, int n, const int32_t* count,
-                             const int32_t* status, cudaStream_t s) {
-  CondHandles hs;
-  for (int i = 0; i < n; ++i) hs.h[i] = h[i];
-  set_conditionals_kernel<<<1, 128, 0, s>>>(hs, n, count, status);
-}
-
 }  // namespace buddy
