@@ -307,7 +307,8 @@ static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, c
   // The first layer feeds the router: its GEMM inputs are kept as bf16 hi + lo
   // pairs so that its output is a continuous function of the inputs.
   const bool split = c.split0 && l == 0;
-  {
+  const bool panel = c.use_tc && c.tc_panel;   // RMSNorms inside the QKV and gate/up GEMMs
+  if (!panel) {
     ProfScope p(c, s, BUDDY_PROF_RMSNORM, 1, prof);
     launch_rmsnorm(c, src, sel, W.attn_norm, c.xn, split ? c.xn_lo : nullptr, s);
   }
@@ -317,6 +318,13 @@ static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, c
   g.split = split;
   g.W = W.w_qkv; g.X = c.xn; g.X_lo = c.xn_lo; g.N = c.qkvN; g.K = c.d; g.out_f32 = c.qkv;
   float* pool = l == 0 ? kv.pool_sum : nullptr;
+  if (panel) {
+    g.in_norm_src = src;
+    g.in_norm_gamma = W.attn_norm;
+    // no RMSNorm kernel in between: the first middle layer's QKV GEMM follows
+    // the compaction kernel that writes its row count
+    g.count_late = l == 1;
+  }
   if (c.use_tc) {
     // bias, RoPE, q, cache append and pool update in the GEMM epilogue
     g.qkv_bias = W.b_qkv; g.kv_len = kv.len; g.kv_seq_off = kv.seq_off; g.kv_cap = kv.cap;
@@ -342,13 +350,17 @@ static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, c
     ProfScope p(c, s, BUDDY_PROF_GEMM_O, 1, prof);
     run_gemm(c, EPI_RESID, g, l, 1, s);
   }
-  {
+  if (!panel) {
     ProfScope p(c, s, BUDDY_PROF_RMSNORM, 1, prof);
     launch_rmsnorm(c, H, sel, W.ffn_norm, c.xn, split ? c.xn_lo : nullptr, s);
   }
   g = GemmArgs{};
   g.sel = sel; g.max_m = sel.n; g.split = split;
   g.W = W.w_gate_up; g.X = c.xn; g.X_lo = c.xn_lo; g.N = c.F; g.K = c.d; g.out_act = c.act;
+  if (panel) {
+    g.in_norm_src = H;
+    g.in_norm_gamma = W.ffn_norm;
+  }
   g.out_act_lo = split ? c.act_lo : nullptr;
   {
     ProfScope p(c, s, BUDDY_PROF_GEMM_GATE_UP, 1, prof);

@@ -74,6 +74,18 @@ struct TcParams {
   float* q_out;
   float* pool;
   int nq, nkv, hd;
+  // Panel mode (at most 8 rows, K a multiple of 64): the activations are the
+  // RMSNorm of the fp32 rows nsrc[rows[j]] (width K), x = bf16(h * rsqrt(
+  // mean(h^2) + neps) * ngamma) (+ remainder), computed by the epilogue warps
+  // into a shared-memory panel holding the unit's K range (two panels, for the
+  // current unit and the next); the ring stages hold weight tiles only.
+  const float* nsrc;
+  const float* ngamma;
+  float neps;
+  int count_late;         // the preceding kernel wrote *count: read it after the wait
+  uint32_t panel_off;     // byte offset of panel 0 in dynamic shared memory
+  uint32_t panel_bytes;   // bytes of one panel (hi, then lo for SPLIT)
+  int panel_kb;           // K blocks one panel holds (hi part)
 };
 
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
@@ -141,6 +153,100 @@ __device__ __forceinline__ void tc_mma_stage(const uint8_t* st, uint32_t d, cons
       ptx::mma_bf16(dt, dx + 2ull * k, dw + 2ull * k, idesc, (!first || k > 0) ? 1u : 0u);
       if (SPLIT) ptx::mma_bf16(dt, dl + 2ull * k, dw + 2ull * k, idesc, 1u);
     }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Panel mode.  Panel layout: K block r of the unit at r * 1024 bytes, rows 0..7
+// of the 128-byte-swizzled K-major tile (rows past m unused); the remainder
+// terms at panel_kb * 1024.  An M = 128 operand read from block r spans the
+// following 15 KiB (later blocks, the next panel, or the tail slack): those
+// rows only feed accumulator rows that are discarded.
+// ---------------------------------------------------------------------------
+// 1 / rms of each row (m <= 8), by the 128 epilogue threads (et = 0..127).
+__device__ __forceinline__ void tc_panel_inv(const TcParams& p, int m, int et, float* red, float* inv) {
+  const int lane = et & 31, w = et >> 5;
+  for (int j = 0; j < m; ++j) {
+    const float* h = p.nsrc + (size_t)(p.rows ? p.rows[j] : j) * p.K;
+    float ss = 0.f;
+    for (int e0 = 0; e0 < p.K; e0 += 16 * 512) {
+      float4 x[16];
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const int e = e0 + (et + k * 128) * 4;
+        x[k] = e < p.K ? *reinterpret_cast<const float4*>(h + e) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int k = 0; k < 16; ++k) ss += x[k].x * x[k].x + x[k].y * x[k].y + x[k].z * x[k].z + x[k].w * x[k].w;
+    }
+    ss = warp_sum(ss);
+    if (lane == 0) red[j * 4 + w] = ss;
+  }
+  epi_bar();
+  if (et < m) inv[et] = rsqrtf(((red[et * 4] + red[et * 4 + 1]) + (red[et * 4 + 2] + red[et * 4 + 3])) / (float)p.K + p.neps);
+  epi_bar();
+}
+
+// The panel of K blocks [kb0, kb1) for rows j < m, then a proxy fence so that
+// the tensor core sees it.  Each thread takes float4 groups (row, column) with
+// all loads issued before the stores.
+template <bool SPLIT>
+__device__ __forceinline__ void tc_panel_write(const TcParams& p, uint8_t* panel, int m, int kb0, int kb1, int et,
+                                               const float* inv) {
+  const int n4 = (kb1 - kb0) * 16;   // float4 groups per row
+  const int total = m * n4;
+  for (int i0 = et; i0 < total; i0 += 4 * 128) {
+    float4 x[4], g[4];
+    int jj[4], qq[4];
+#pragma unroll
+    for (int b = 0; b < 4; ++b) {
+      const int i = i0 + b * 128;
+      jj[b] = i < total ? i / n4 : -1;
+      qq[b] = i - (jj[b] < 0 ? 0 : jj[b]) * n4;
+      if (jj[b] >= 0) {
+        const int c = kb0 * kTileK + qq[b] * 4;
+        x[b] = *reinterpret_cast<const float4*>(p.nsrc + (size_t)(p.rows ? p.rows[jj[b]] : jj[b]) * p.K + c);
+        g[b] = *reinterpret_cast<const float4*>(p.ngamma + c);
+      }
+    }
+#pragma unroll
+    for (int b = 0; b < 4; ++b) {
+      if (jj[b] < 0) continue;
+      const int j = jj[b], r = qq[b] >> 4, q = qq[b] & 15;
+      const float iv = inv[j];
+      const float y[4] = {x[b].x * iv * g[b].x, x[b].y * iv * g[b].y, x[b].z * iv * g[b].z, x[b].w * iv * g[b].w};
+      uint32_t hi[2], lo[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const bf16 a = from_f<bf16>(y[2 * u]), c2 = from_f<bf16>(y[2 * u + 1]);
+        hi[u] = (uint32_t)__bfloat16_as_ushort(a) | ((uint32_t)__bfloat16_as_ushort(c2) << 16);
+        if (SPLIT) {
+          const bf16 la = from_f<bf16>(y[2 * u] - to_f(a)), lc = from_f<bf16>(y[2 * u + 1] - to_f(c2));
+          lo[u] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lc) << 16);
+        }
+      }
+      // row j of K block r: 16-byte chunk q / 2 of the row at chunk (q / 2) ^ j
+      const uint32_t off = (uint32_t)r * 1024u + (uint32_t)j * 128u + (uint32_t)((((q >> 1) ^ j) & 7) << 4) +
+                           (uint32_t)((q & 1) * 8);
+      *reinterpret_cast<uint2*>(panel + off) = make_uint2(hi[0], hi[1]);
+      if (SPLIT) *reinterpret_cast<uint2*>(panel + (size_t)p.panel_kb * 1024 + off) = make_uint2(lo[0], lo[1]);
+    }
+  }
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// MMAs of one stage in panel mode: weights from the stage, activations (one
+// M-tile, and SPLIT the remainder terms) from panel block `pb`.
+template <bool SPLIT>
+__device__ __forceinline__ void tc_mma_panel(const uint8_t* st, const uint8_t* pb, uint32_t d, const TcParams& p,
+                                             uint32_t idesc, bool first) {
+  const uint64_t dw = ptx::smem_desc_sw128(st);
+  const uint64_t dx = ptx::smem_desc_sw128(pb);
+  const uint64_t dl = ptx::smem_desc_sw128(pb + (size_t)p.panel_kb * 1024);
+#pragma unroll
+  for (int k = 0; k < kTileK / 16; ++k) {
+    ptx::mma_bf16(d, dx + 2ull * k, dw + 2ull * k, idesc, (!first || k > 0) ? 1u : 0u);
+    if (SPLIT) ptx::mma_bf16(d, dl + 2ull * k, dw + 2ull * k, idesc, 1u);
   }
 }
 

@@ -36,23 +36,31 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                    const __grid_constant__ CUtensorMap txlo, const TcParams p) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kTcMaxStages], empty_bar[kTcMaxStages];
-  __shared__ __align__(8) uint64_t tfull_bar[2], tempty_bar[2], done_bar;
+  __shared__ __align__(8) uint64_t tfull_bar[2], tempty_bar[2], done_bar, pfull_bar[2];
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
   __shared__ volatile int consumed;
   __shared__ int last_flag;
+  __shared__ float pred[32], pinv[8];   // panel mode: sums of squares, 1 / rms per row
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
 
   // A layer that no row selected leaves before any setup.  Its row count was
-  // written by the compaction kernel, which completed before the preceding
-  // kernel of the step let this one launch (every kernel of the step waits on
-  // its predecessor before allowing its dependents to start), so it may be read
-  // before the wait.  The wait itself still happens, so that the completion of
-  // this kernel implies the completion of everything enqueued before it.
-  if (p.count && *reinterpret_cast<const volatile int32_t*>(p.count) <= 0) {
+  // written by the compaction kernel; unless that kernel is the one enqueued
+  // right before this GEMM (count_late), it completed before the preceding
+  // kernel let this one launch (every kernel of the step waits on its
+  // predecessor before allowing its dependents to start), so the count may be
+  // read before the wait.  The wait itself always happens, so that the
+  // completion of this kernel implies the completion of everything enqueued
+  // before it.
+  bool waited = false;
+  if (p.count_late) {
     pdl_wait();
+    waited = true;
+  }
+  if (p.count && *reinterpret_cast<const volatile int32_t*>(p.count) <= 0) {
+    if (!waited) pdl_wait();
     pdl_trigger();
     return;
   }
@@ -67,6 +75,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       ptx::mbar_init(&tempty_bar[a], 4);
     }
     ptx::mbar_init(&done_bar, 1);
+    ptx::mbar_init(&pfull_bar[0], 1);
+    ptx::mbar_init(&pfull_bar[1], 1);
     abort_flag = 0;
     consumed = 0;
     ptx::fence_mbar_init();
@@ -99,7 +109,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       }
     }
   }
-  pdl_wait();
+  if (!waited) pdl_wait();
   pdl_trigger();
   const int m = call_aborted(p.status) ? 0 : (p.count ? *p.count : p.n);
   if (m <= 0) {
@@ -118,7 +128,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (warp == 1) ptx::tmem_dealloc(tmem_base, p.tmem_cols);
     return;
   }
-  const uint32_t x_bytes = tc_x_bytes(m, SPLIT);
+  const bool panel = p.nsrc != nullptr;
+  const uint32_t x_bytes = panel ? 0u : tc_x_bytes(m, SPLIT);
   const uint32_t acc_cols = (uint32_t)(p.mt * p.bw);
 
   if (warp == 0) {
@@ -135,7 +146,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           uint8_t* st = smem + (size_t)stage * p.stage_bytes;
           if (issued < npre) {
             // weight tile already in flight: add the activation tiles
-            ptx::mbar_arrive_expect_tx(&full_bar[stage], x_bytes);
+            if (panel) ptx::mbar_arrive(&full_bar[stage]);
+            else ptx::mbar_arrive_expect_tx(&full_bar[stage], x_bytes);
           } else {
             if (!ptx::mbar_wait_bounded(&empty_bar[stage], ph ^ 1u, kWaitLimitNs, &abort_flag)) {
               ok = false;
@@ -144,7 +156,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             ptx::mbar_arrive_expect_tx(&full_bar[stage], w_bytes + x_bytes);
             tc_load_w<EPI>(st, &tw, &full_bar[stage], p, tile, kb, pol);
           }
-          tc_load_x<SPLIT>(st, &tx, &txlo, &full_bar[stage], p, m, kb);
+          if (!panel) tc_load_x<SPLIT>(st, &tx, &txlo, &full_bar[stage], p, m, kb);
           ++issued;
           if (++stage == p.stages) {
             stage = 0;
@@ -167,14 +179,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       uint32_t ph = 0;
       int acc = 0;
       uint32_t acc_ph = 0;
-      int n_consumed = 0;
+      int n_consumed = 0, ui = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x) {
+      for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x, ++ui) {
         const int split = u / p.n_tiles;
         const int kb0 = split * p.kb_per_split, kb1 = min(p.kb_total, kb0 + p.kb_per_split);
         if (!ptx::mbar_wait_bounded(&tempty_bar[acc], acc_ph ^ 1u, kWaitLimitNs, &abort_flag)) break;
+        if (panel &&
+            !ptx::mbar_wait_bounded(&pfull_bar[ui & 1], (uint32_t)((ui >> 1) & 1), kWaitLimitNs, &abort_flag))
+          break;
         ptx::tc_fence_after();
         const uint32_t d = tmem_base + (uint32_t)acc * acc_cols;
+        const uint8_t* pan = smem + p.panel_off + (size_t)(ui & 1) * p.panel_bytes;
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!ptx::mbar_wait_bounded(&full_bar[stage], ph, kWaitLimitNs, &abort_flag)) {
             ok = false;
@@ -182,7 +198,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           }
           consumed = ++n_consumed;
           ptx::tc_fence_after();
-          tc_mma_stage<SPLIT>(smem + (size_t)stage * p.stage_bytes, d, p, m, idesc, kb == kb0);
+          if (panel)
+            tc_mma_panel<SPLIT>(smem + (size_t)stage * p.stage_bytes, pan + (size_t)(kb - kb0) * 1024, d, p, idesc,
+                                kb == kb0);
+          else
+            tc_mma_stage<SPLIT>(smem + (size_t)stage * p.stage_bytes, d, p, m, idesc, kb == kb0);
           ptx::mma_commit(&empty_bar[stage]);
           if (++stage == p.stages) {
             stage = 0;
@@ -208,7 +228,29 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // ------------------------------------------------------------- epilogue
     int acc = 0;
     uint32_t acc_ph = 0;
-    for (int u = blockIdx.x; u < p.units; u += gridDim.x) {
+    const int et = threadIdx.x - 64;
+    if (panel && blockIdx.x < p.units) {
+      // the norm of every row, then the first unit's panel
+      tc_panel_inv(p, m, et, pred, pinv);
+      const int split = blockIdx.x / p.n_tiles;
+      const int kb0 = split * p.kb_per_split, kb1 = min(p.kb_total, kb0 + p.kb_per_split);
+      tc_panel_write<SPLIT>(p, smem + p.panel_off, m, kb0, kb1, et, pinv);
+      epi_bar();
+      if (et == 0) ptx::mbar_arrive(&pfull_bar[0]);
+    }
+    int ui = 0;
+    for (int u = blockIdx.x; u < p.units; u += gridDim.x, ++ui) {
+      const int un = u + gridDim.x;
+      if (panel && un < p.units) {
+        // the next unit's panel goes into the buffer the unit before this one
+        // used (its MMAs completed: its accumulator was drained)
+        const int split = un / p.n_tiles;
+        const int kb0 = split * p.kb_per_split, kb1 = min(p.kb_total, kb0 + p.kb_per_split);
+        tc_panel_write<SPLIT>(p, smem + p.panel_off + (size_t)((ui + 1) & 1) * p.panel_bytes, m, kb0, kb1, et,
+                              pinv);
+        epi_bar();
+        if (et == 0) ptx::mbar_arrive(&pfull_bar[(ui + 1) & 1]);
+      }
       const bool ok = ptx::mbar_wait_bounded(&tfull_bar[acc], acc_ph, kWaitLimitNs, &abort_flag);
       if (epi_bar_any(!ok)) break;
       ptx::tc_fence_after();
@@ -368,6 +410,26 @@ int gemm_tc_prepare(Ctx& c) {
     c.gemm_ctr_n = max_tiles;
   }
   if (cudaMemset(c.gemm_ctr, 0, c.gemm_ctr_n * sizeof(int32_t)) != cudaSuccess) return BUDDY_ERR_CUDA;
+  // Panel mode for up to eight rows: the QKV and gate/up GEMMs normalise their
+  // own activations (no RMSNorm kernels, no activation copies).  Stages hold
+  // weight tiles only; two panels of the largest K range follow the ring, then
+  // 15 KiB for the tail of an M = 128 operand read.
+  c.tc_panel = c.maxB <= 8 && c.d % kTileK == 0;
+  if (c.tc_panel) {
+    int N, K, tiles;
+    gemm_shape(c, 0, &N, &K, &tiles);
+    c.tc_panel_kb = (K / kTileK + c.tc_splits[0] - 1) / c.tc_splits[0];
+    gemm_shape(c, 2, &N, &K, &tiles);
+    c.tc_panel_kb = std::max(c.tc_panel_kb, (K / kTileK + c.tc_splits[2] - 1) / c.tc_splits[2]);
+    const int limit = 227 * 1024 - 2 * 1024;
+    for (int v = 0; v < 2; ++v) {
+      c.tc_panel_bytes[v] = (uint32_t)(v + 1) * (uint32_t)c.tc_panel_kb * 1024u;
+      const int fixed = 1024 + 2 * (int)c.tc_panel_bytes[v] + 15 * 1024;
+      c.tc_pstages[v] = std::min(kTcMaxStages, (limit - fixed) / (c.tc_bw * 128));
+      c.tc_psmem[v] = c.tc_pstages[v] * c.tc_bw * 128 + fixed;
+      if (c.tc_pstages[v] < 3) c.tc_panel = false;
+    }
+  }
   const char* lk_env = getenv("BUDDY_LAYER_KERNEL");
   c.use_lk = layer_kernel_supported(c) && lk_env && lk_env[0] == '1';   // opt-in
   if (c.use_lk && !c.lk_bar) {
@@ -375,14 +437,16 @@ int gemm_tc_prepare(Ctx& c) {
     if (cudaMemset(c.lk_bar, 0, 2 * sizeof(unsigned)) != cudaSuccess) return BUDDY_ERR_CUDA;
   }
   const cudaFuncAttribute A = cudaFuncAttributeMaxDynamicSharedMemorySize;
+  const int qs0 = std::max(c.tc_smem[0], c.tc_panel ? c.tc_psmem[0] : 0);
+  const int qs1 = std::max(c.tc_smem[1], c.tc_panel ? c.tc_psmem[1] : 0);
   if (cudaFuncSetAttribute(gemm_tc_kernel<EPI_STORE_F32, false>, A, c.tc_smem[0]) ||
       cudaFuncSetAttribute(gemm_tc_kernel<EPI_RESID, false>, A, c.tc_smem[0]) ||
-      cudaFuncSetAttribute(gemm_tc_kernel<EPI_SWIGLU, false>, A, c.tc_smem[0]) ||
+      cudaFuncSetAttribute(gemm_tc_kernel<EPI_SWIGLU, false>, A, qs0) ||
       cudaFuncSetAttribute(gemm_tc_kernel<EPI_STORE_F32, true>, A, c.tc_smem[1]) ||
       cudaFuncSetAttribute(gemm_tc_kernel<EPI_RESID, true>, A, c.tc_smem[1]) ||
-      cudaFuncSetAttribute(gemm_tc_kernel<EPI_SWIGLU, true>, A, c.tc_smem[1]) ||
-      cudaFuncSetAttribute(gemm_tc_kernel<EPI_QKV, false>, A, c.tc_smem[0]) ||
-      cudaFuncSetAttribute(gemm_tc_kernel<EPI_QKV, true>, A, c.tc_smem[1]))
+      cudaFuncSetAttribute(gemm_tc_kernel<EPI_SWIGLU, true>, A, qs1) ||
+      cudaFuncSetAttribute(gemm_tc_kernel<EPI_QKV, false>, A, qs0) ||
+      cudaFuncSetAttribute(gemm_tc_kernel<EPI_QKV, true>, A, qs1))
     return BUDDY_ERR_CUDA;
   return BUDDY_OK;
 }
@@ -430,6 +494,20 @@ void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s) {
   p.vc = (bf16*)a.vc;
   p.q_out = a.q_out;
   p.pool = a.pool;
+  size_t smem = c.tc_smem[v];
+  if (a.in_norm_src) {   // panel mode
+    p.nsrc = a.in_norm_src;
+    p.ngamma = a.in_norm_gamma;
+    p.neps = c.cfg.rms_eps;
+    p.stages = c.tc_pstages[v];
+    p.stage_bytes = (uint32_t)c.tc_bw * 128u;
+    p.w_off = 0;
+    p.panel_off = (uint32_t)p.stages * p.stage_bytes;
+    p.panel_bytes = c.tc_panel_bytes[v];
+    p.panel_kb = c.tc_panel_kb;
+    smem = c.tc_psmem[v];
+  }
+  p.count_late = a.count_late ? 1 : 0;
   p.nq = c.nq;
   p.nkv = c.nkv;
   p.hd = c.hd;
@@ -438,7 +516,7 @@ void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s) {
   const CUtensorMap& tx = c.tmaps_host[(size_t)c.L * 4 + xi];
   const CUtensorMap& txlo = c.tmaps_host[(size_t)c.L * 4 + 3 + xi];
   const int grid = std::min(p.units, c.num_sms);
-  const size_t smem = c.tc_smem[v];
+
   if (a.split) {
     switch (epi) {
       case EPI_QKV:

@@ -59,6 +59,11 @@ struct GemmArgs {
   const int32_t* status;
   int layer;              // tensor-core path: which layer's weight map
   int which;              // 0 qkv, 1 o, 2 gate_up, 3 down
+  // tensor-core path, small batches: X = RMSNorm(in_norm_src[rows]) computed
+  // inside the GEMM (panel mode; X and X_lo unused)
+  const float* in_norm_src;
+  const float* in_norm_gamma;
+  bool count_late;        // the kernel enqueued just before wrote *sel.count
 };
 
 struct Ctx;
@@ -173,6 +178,10 @@ struct Ctx {
   size_t gemm_ws_elems = 0;
   int32_t* gemm_ctr = nullptr;
   int gemm_ctr_n = 0;
+  // panel mode: the RMSNorms before the QKV and gate/up GEMMs run inside them
+  bool tc_panel = false;
+  int tc_panel_kb = 0, tc_pstages[2] = {1, 1}, tc_psmem[2] = {0, 0};
+  uint32_t tc_panel_bytes[2] = {0, 0};
 
   // profiler: event pairs around kernel launches (direct-launch mode only)
   int profiling = 0;
