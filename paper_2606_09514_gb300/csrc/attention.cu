@@ -19,10 +19,43 @@
 #include <algorithm>
 
 #include "attn_common.cuh"
+#include "attn_tc.cuh"
 #include "common.cuh"
 #include "internal.h"
 
 namespace buddy {
+
+template <int HD, bool SPLIT>
+__global__ void __launch_bounds__(kTcaThreads) attn_tc_kernel(AttnArgs<bf16> A) {
+  extern __shared__ __align__(16) uint8_t smraw[];
+  __shared__ float sc[32];
+  attn_tc_run<HD, SPLIT>(A, blockIdx.x, gridDim.x, smraw, sc, true);
+}
+
+// bf16 caches with at most 8 query heads per KV head: the tensor-core loop
+template <int HD, bool SPLIT>
+static void attn_tc_impl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q, void* out,
+                         void* out_lo, cudaStream_t s) {
+  const size_t smem = attn_tc_smem_bytes(HD, c.maxB);
+  static bool attr_set = false;   // one per instantiation
+  static int occ = 0;
+  static size_t occ_smem = 0;
+  if (!attr_set) {
+    cudaFuncSetAttribute(attn_tc_kernel<HD, SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+    attr_set = true;
+  }
+  if (occ == 0 || occ_smem != smem) {
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, attn_tc_kernel<HD, SPLIT>, kTcaThreads, smem) !=
+        cudaSuccess)
+      occ = 1;
+    occ_smem = smem;
+  }
+  const int grid = c.num_sms * std::max(1, std::min(occ, 4));
+  AttnArgs<bf16> A{q, sel.rows, sel.count, sel.n, c.nq, c.nkv, kv.len, kv.seq_off, kv.cap,
+                   (const bf16*)kv.k_cache[layer], (const bf16*)kv.v_cache[layer], c.attn_max_chunks, c.attn_m,
+                   c.attn_l, c.attn_acc, c.attn_ctr, (bf16*)out, (bf16*)out_lo, c.status};
+  launch_k(attn_tc_kernel<HD, SPLIT>, grid, kTcaThreads, smem, s, c.pdl, A);
+}
 
 template <typename T, int HD, int GP>
 __global__ void __launch_bounds__(kAttnThreads) attn_kernel(AttnArgs<T> A) {
@@ -73,7 +106,15 @@ int attention_chunk() { return kChunk; }
 
 void launch_attention(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q,
                       void* out, void* out_lo, cudaStream_t s) {
-  if (c.dtype == BUDDY_DTYPE_BF16) {
+  if (c.dtype == BUDDY_DTYPE_BF16 && c.nq / c.nkv <= 8) {
+    if (c.hd == 128) {
+      if (out_lo) attn_tc_impl<128, true>(c, sel, kv, layer, q, out, out_lo, s);
+      else attn_tc_impl<128, false>(c, sel, kv, layer, q, out, out_lo, s);
+    } else {
+      if (out_lo) attn_tc_impl<64, true>(c, sel, kv, layer, q, out, out_lo, s);
+      else attn_tc_impl<64, false>(c, sel, kv, layer, q, out, out_lo, s);
+    }
+  } else if (c.dtype == BUDDY_DTYPE_BF16) {
     if (c.hd == 128) attn_group<bf16, 128>(c, sel, kv, layer, q, out, out_lo, s);
     else attn_group<bf16, 64>(c, sel, kv, layer, q, out, out_lo, s);
   } else {

@@ -98,6 +98,86 @@ inline size_t attn_smem_bytes(size_t fixed, int G, int hd, int max_spans, int ma
          (size_t)max_rows * 16;
 }
 
+// Merge of a (row j, KV head g)'s nsp span partials, by the CTA that
+// completed it (NT threads numbered tid), in span order: the tpo adjacent
+// threads of an output (four consecutive channels of one head) take spans
+// sub, sub + tpo, ... with a running rescaled sum (running max M, sum L, output
+// a), loading D of their spans' partials at a time; the tpo results are then
+// combined by a lane butterfly (every thread ends with the same values).  When
+// the outputs outnumber the threads, the threads take them in rounds of NT.
+template <typename T, int HD, int NT>
+__device__ __forceinline__ void attn_span_merge(const AttnArgs<T>& A, int j, int g, int nsp, size_t obase, int tid) {
+  constexpr int D = NT >= 256 ? 16 : 8;   // partials in flight per thread
+  const int nq = A.nq, G = A.nq / A.nkv, max_spans = A.max_spans;
+  const float* __restrict__ part_acc = A.part_acc;
+  const float* __restrict__ part_m = A.part_m;
+  const float* __restrict__ part_l = A.part_l;
+  T* __restrict__ out = A.out;
+  T* __restrict__ out_lo = A.out_lo;
+  const int n4 = G * HD / 4;
+  int tpo = 1;
+  while (tpo < 8 && tpo * 2 * n4 <= NT) tpo *= 2;
+  const int nwork = (n4 * tpo + 31) & ~31;   // whole warps take part in the butterfly
+  constexpr int kRounds = (8 * HD / 4 + NT - 1) / NT;   // at most 8 query heads per KV head
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const int w = tid + r * NT;
+    if (w >= nwork) break;
+    const int x4 = w / tpo, sub = w % tpo;
+    const bool act = x4 < n4;
+    const int h = act ? (x4 * 4) / HD : 0, ee = act ? x4 * 4 - h * HD : 0;
+    const size_t hb = ((size_t)j * nq + g * G + h) * max_spans;
+    float M = -INFINITY, L = 0.f;
+    float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int c0 = sub; act && c0 < nsp; c0 += D * tpo) {
+      float4 t[D];
+      float ms[D], ls[D];
+#pragma unroll
+      for (int k = 0; k < D; ++k) {
+        const int cc = c0 + k * tpo;
+        if (cc < nsp) {
+          t[k] = __ldcg(reinterpret_cast<const float4*>(part_acc + (hb + cc) * HD + ee));
+          ms[k] = __ldcg(part_m + hb + cc);
+          ls[k] = __ldcg(part_l + hb + cc);
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < D; ++k) {
+        if (c0 + k * tpo < nsp) {
+          const float mn = fmaxf(M, ms[k]);
+          const float fo = expf(M - mn), fn = expf(ms[k] - mn);
+          a.x = a.x * fo + t[k].x * fn;
+          a.y = a.y * fo + t[k].y * fn;
+          a.z = a.z * fo + t[k].z * fn;
+          a.w = a.w * fo + t[k].w * fn;
+          L = L * fo + ls[k] * fn;
+          M = mn;
+        }
+      }
+    }
+    for (int o = 1; o < tpo; o <<= 1) {
+      const float M2 = __shfl_xor_sync(0xffffffffu, M, o), L2 = __shfl_xor_sync(0xffffffffu, L, o);
+      const float ax = __shfl_xor_sync(0xffffffffu, a.x, o), ay = __shfl_xor_sync(0xffffffffu, a.y, o);
+      const float az = __shfl_xor_sync(0xffffffffu, a.z, o), aw = __shfl_xor_sync(0xffffffffu, a.w, o);
+      const float mn = fmaxf(M, M2);
+      const float f1 = M == -INFINITY ? 0.f : expf(M - mn), f2 = M2 == -INFINITY ? 0.f : expf(M2 - mn);
+      a.x = a.x * f1 + ax * f2;
+      a.y = a.y * f1 + ay * f2;
+      a.z = a.z * f1 + az * f2;
+      a.w = a.w * f1 + aw * f2;
+      L = L * f1 + L2 * f2;
+      M = mn;
+    }
+    if (act && sub == 0) {
+      const size_t o = obase + (size_t)h * HD + ee;
+      store_out(out, out_lo, o + 0, a.x / L);
+      store_out(out, out_lo, o + 1, a.y / L);
+      store_out(out, out_lo, o + 2, a.z / L);
+      store_out(out, out_lo, o + 3, a.w / L);
+    }
+  }
+}
+
 // Query heads per KV head rounded up to 1, 2, 4 or 8 (the work-loop template).
 inline int attn_group_pad(int G) { return G <= 1 ? 1 : (G <= 2 ? 2 : (G <= 4 ? 4 : 8)); }
 
@@ -456,70 +536,7 @@ __device__ __forceinline__ void attn_run(const AttnArgs<T>& A, int tid, int cta,
         __threadfence();
       }
       sync();
-      if (*last_s_p) {
-        // merge: the tpo adjacent threads of an output (four consecutive
-        // channels of one head) take spans sub, sub + tpo, ... with a running
-        // rescaled sum (running max M, sum L, output a), loading sixteen of
-        // their spans' partials at a time; the tpo results are then combined
-        // by a lane butterfly (every thread ends with the same values)
-        const int n4 = G * HD / 4;
-        int tpo = 1;
-        while (tpo < 8 && tpo * 2 * n4 <= NT) tpo *= 2;
-        const int x4 = tid / tpo, sub = tid % tpo;
-        if (tid < ((n4 * tpo + 31) & ~31)) {   // whole warps take part in the butterfly
-          const bool act = x4 < n4;
-          const int h = act ? (x4 * 4) / HD : 0, ee = act ? x4 * 4 - h * HD : 0;
-          const size_t hb = ((size_t)j * nq + g * G + h) * max_spans;
-          float M = -INFINITY, L = 0.f;
-          float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-          for (int c0 = sub; act && c0 < nsp; c0 += 16 * tpo) {
-            float4 t[16];
-            float ms[16], ls[16];
-#pragma unroll
-            for (int k = 0; k < 16; ++k) {
-              const int cc = c0 + k * tpo;
-              if (cc < nsp) {
-                t[k] = __ldcg(reinterpret_cast<const float4*>(part_acc + (hb + cc) * HD + ee));
-                ms[k] = __ldcg(part_m + hb + cc);
-                ls[k] = __ldcg(part_l + hb + cc);
-              }
-            }
-#pragma unroll
-            for (int k = 0; k < 16; ++k) {
-              if (c0 + k * tpo < nsp) {
-                const float mn = fmaxf(M, ms[k]);
-                const float fo = expf(M - mn), fn = expf(ms[k] - mn);
-                a.x = a.x * fo + t[k].x * fn;
-                a.y = a.y * fo + t[k].y * fn;
-                a.z = a.z * fo + t[k].z * fn;
-                a.w = a.w * fo + t[k].w * fn;
-                L = L * fo + ls[k] * fn;
-                M = mn;
-              }
-            }
-          }
-          for (int o = 1; o < tpo; o <<= 1) {
-            const float M2 = __shfl_xor_sync(0xffffffffu, M, o), L2 = __shfl_xor_sync(0xffffffffu, L, o);
-            const float ax = __shfl_xor_sync(0xffffffffu, a.x, o), ay = __shfl_xor_sync(0xffffffffu, a.y, o);
-            const float az = __shfl_xor_sync(0xffffffffu, a.z, o), aw = __shfl_xor_sync(0xffffffffu, a.w, o);
-            const float mn = fmaxf(M, M2);
-            const float f1 = M == -INFINITY ? 0.f : expf(M - mn), f2 = M2 == -INFINITY ? 0.f : expf(M2 - mn);
-            a.x = a.x * f1 + ax * f2;
-            a.y = a.y * f1 + ay * f2;
-            a.z = a.z * f1 + az * f2;
-            a.w = a.w * f1 + aw * f2;
-            L = L * f1 + L2 * f2;
-            M = mn;
-          }
-          if (act && sub == 0) {
-            const size_t o = obase + (size_t)h * HD + ee;
-            store_out(out, out_lo, o + 0, a.x / L);
-            store_out(out, out_lo, o + 1, a.y / L);
-            store_out(out, out_lo, o + 2, a.z / L);
-            store_out(out, out_lo, o + 3, a.w / L);
-          }
-        }
-      }
+      if (*last_s_p) attn_span_merge<T, HD, NT>(A, j, g, nsp, obase, tid);
     }
     sync();
   }
