@@ -314,7 +314,7 @@ def run_ours(args, ws, rank, local):
     per_class_bytes = class_bytes(s, prof_masks, prof_ctx, B)
     roof = None
     if dom in per_class_bytes and prof[dom][1] > 0:
-        launches = prof[dom][1] if dom != "attention" else prof[dom][1] // 2
+        launches = prof[dom][1]
         bytes_per_launch = per_class_bytes[dom] / launches
         avg_s = prof[dom][0] / 1e3 / launches
         ach = bytes_per_launch / avg_s / 1e9
@@ -329,8 +329,8 @@ def run_ours(args, ws, rank, local):
     # the timed steps launch every middle layer (a layer no row selected exits
     # at once); the profiled steps launch only the selected ones
     per_layer = ("rmsnorm", "gemm_qkv", "qkv_finalize", "attention", "gemm_o", "gemm_gate_up", "gemm_down",
-                 "layer")
-    exec_layers = (prof.get("gemm_gate_up", (0, 0))[1] + prof.get("layer", (0, 0))[1]) / prof_steps
+                 "layer", "gemm_fixup")
+    exec_layers = (prof.get("attention", (0, 0))[1] + prof.get("layer", (0, 0))[1]) / prof_steps
     per_layer_kernels = sum(prof.get(k, (0, 0))[1] for k in per_layer) / max(exec_layers * prof_steps, 1)
     graph_extra = max(s.n_layers - exec_layers, 0) * per_layer_kernels
     out = {

@@ -225,6 +225,7 @@ enum {
   BUDDY_PROF_ATTENTION, BUDDY_PROF_GEMM_O, BUDDY_PROF_GEMM_GATE_UP, BUDDY_PROF_GEMM_DOWN,
   BUDDY_PROF_ROUTE, BUDDY_PROF_COMPACT, BUDDY_PROF_OTHER,
   BUDDY_PROF_LAYER,   /* a whole block as one persistent kernel (small batches) */
+  BUDDY_PROF_GEMM_FIXUP,   /* split-K sums + epilogues of the GEMMs (larger batches) */
   BUDDY_PROF_NCLASS
 };
 

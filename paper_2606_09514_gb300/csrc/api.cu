@@ -254,7 +254,7 @@ extern "C" int buddy_set_profiling(buddy_ctx* ctx, int32_t on) {
 extern "C" const char* buddy_profile_class_name(int32_t cls) {
   static const char* names[BUDDY_PROF_NCLASS] = {"check", "rmsnorm", "gemm_qkv", "qkv_finalize",
                                                  "attention", "gemm_o", "gemm_gate_up", "gemm_down",
-                                                 "route", "compact", "other", "layer"};
+                                                 "route", "compact", "other", "layer", "gemm_fixup"};
   return (cls >= 0 && cls < BUDDY_PROF_NCLASS) ? names[cls] : "unknown";
 }
 
@@ -283,13 +283,21 @@ extern "C" int buddy_profile_read(buddy_ctx* ctx, int32_t n_cls, float* ms, int3
 // ---------------------------------------------------------------------------
 // GEMM dispatch
 // ---------------------------------------------------------------------------
-static void run_gemm(const Ctx& c, int epi, GemmArgs a, int layer, int which, cudaStream_t s) {
+static void run_gemm(Ctx& c, int epi, GemmArgs a, int layer, int which, cudaStream_t s, int cls, bool prof) {
   a.status = c.status;
   a.layer = layer;
   a.which = which;
   if (c.use_tc) {
-    launch_gemm_tc(c, epi, a, s);
+    {
+      ProfScope p(c, s, cls, 1, prof);
+      launch_gemm_tc(c, epi, a, s);
+    }
+    if (c.tc_defer) {
+      ProfScope p(c, s, BUDDY_PROF_GEMM_FIXUP, 1, prof);
+      launch_gemm_fix(c, epi, a, s);
+    }
   } else {
+    ProfScope p(c, s, cls, 1, prof);
     launch_gemm_simt(c, epi, a, s);
   }
 }
@@ -329,27 +337,20 @@ static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, c
     // bias, RoPE, q, cache append and pool update in the GEMM epilogue
     g.qkv_bias = W.b_qkv; g.kv_len = kv.len; g.kv_seq_off = kv.seq_off; g.kv_cap = kv.cap;
     g.kc = kv.k_cache[l]; g.vc = kv.v_cache[l]; g.q_out = c.q; g.pool = pool;
-    ProfScope p(c, s, BUDDY_PROF_GEMM_QKV, 1, prof);
-    run_gemm(c, EPI_QKV, g, l, 0, s);
+    run_gemm(c, EPI_QKV, g, l, 0, s, BUDDY_PROF_GEMM_QKV, prof);
   } else {
-    {
-      ProfScope p(c, s, BUDDY_PROF_GEMM_QKV, 1, prof);
-      run_gemm(c, EPI_STORE_F32, g, l, 0, s);
-    }
+    run_gemm(c, EPI_STORE_F32, g, l, 0, s, BUDDY_PROF_GEMM_QKV, prof);
     ProfScope p(c, s, BUDDY_PROF_QKV_FINALIZE, 1, prof);
     launch_qkv_finalize(c, c.qkv, W.b_qkv, sel, kv, l, c.q, pool, s);
   }
   {
-    ProfScope p(c, s, BUDDY_PROF_ATTENTION, 2, prof);
+    ProfScope p(c, s, BUDDY_PROF_ATTENTION, 1, prof);
     launch_attention(c, sel, kv, l, c.q, c.attn_out, split ? c.attn_lo : nullptr, s);
   }
   g = GemmArgs{};
   g.sel = sel; g.max_m = sel.n; g.split = split;
   g.W = W.w_o; g.X = c.attn_out; g.X_lo = c.attn_lo; g.N = c.d; g.K = c.qd; g.resid_src = src; g.resid_dst = H;
-  {
-    ProfScope p(c, s, BUDDY_PROF_GEMM_O, 1, prof);
-    run_gemm(c, EPI_RESID, g, l, 1, s);
-  }
+  run_gemm(c, EPI_RESID, g, l, 1, s, BUDDY_PROF_GEMM_O, prof);
   if (!panel) {
     ProfScope p(c, s, BUDDY_PROF_RMSNORM, 1, prof);
     launch_rmsnorm(c, H, sel, W.ffn_norm, c.xn, split ? c.xn_lo : nullptr, s);
@@ -362,17 +363,11 @@ static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, c
     g.in_norm_gamma = W.ffn_norm;
   }
   g.out_act_lo = split ? c.act_lo : nullptr;
-  {
-    ProfScope p(c, s, BUDDY_PROF_GEMM_GATE_UP, 1, prof);
-    run_gemm(c, EPI_SWIGLU, g, l, 2, s);
-  }
+  run_gemm(c, EPI_SWIGLU, g, l, 2, s, BUDDY_PROF_GEMM_GATE_UP, prof);
   g = GemmArgs{};
   g.sel = sel; g.max_m = sel.n; g.split = split;
   g.W = W.w_down; g.X = c.act; g.X_lo = c.act_lo; g.N = c.d; g.K = c.F; g.resid_src = H; g.resid_dst = H;
-  {
-    ProfScope p(c, s, BUDDY_PROF_GEMM_DOWN, 1, prof);
-    run_gemm(c, EPI_RESID, g, l, 3, s);
-  }
+  run_gemm(c, EPI_RESID, g, l, 3, s, BUDDY_PROF_GEMM_DOWN, prof);
 }
 
 struct StepIO {

@@ -41,6 +41,8 @@ constexpr int kTileK = 64;                       // K columns per stage (128 B o
 constexpr uint32_t kXTileMax = 128 * 128;        // bytes one M-tile operand spans
 constexpr int kTileN = 256;                      // weight rows per tile (MMA N)
 constexpr uint64_t kWaitLimitNs = 4000000000ull; // 4 s
+constexpr int kTcFixThreads = 256;                // deferred-fixup kernel
+constexpr int kTcDeferRows = 8;                   // larger batches defer the split-K fixup
 
 struct TcParams {
   int N, K;
@@ -86,6 +88,9 @@ struct TcParams {
   uint32_t panel_off;     // byte offset of panel 0 in dynamic shared memory
   uint32_t panel_bytes;   // bytes of one panel (hi, then lo for SPLIT)
   int panel_kb;           // K blocks one panel holds (hi part)
+  // Deferred fixup: units only stage their partials; a second kernel
+  // (gemm_fix_kernel) sums the splits and applies the epilogue on every SM.
+  int defer;
 };
 
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
@@ -355,6 +360,44 @@ __device__ __forceinline__ void tc_apply4(const TcParams& p, int tile, int j, in
   }
 }
 
+// One epilogue item (row j, 4-column group at c of `tile`): the partials of
+// all K splits (and of the partner columns) are summed in split order, eight
+// splits' loads in flight at a time, and the epilogue is applied.
+template <int EPI, bool SPLIT>
+__device__ __forceinline__ void tc_fix_item(const TcParams& p, int tile, int j, int c) {
+  const int po = tc_partner_off<EPI>(p);
+  const size_t sstride = (size_t)p.n_tiles * p.rows_max * p.bw;   // one split's slots
+  const float* sl = p.ws + ((size_t)tile * p.rows_max + j) * p.bw + c;
+  float v[4] = {0.f, 0.f, 0.f, 0.f}, vp[4] = {0.f, 0.f, 0.f, 0.f}, rs[4] = {0.f, 0.f, 0.f, 0.f};
+  if (EPI == EPI_RESID) {
+    const int seq = p.rows ? p.rows[j] : j;
+    const int n0 = tile * p.bw + c;
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (n0 + i < p.N) rs[i] = p.resid_src[(size_t)seq * p.N + n0 + i];
+  }
+  for (int s0 = 0; s0 < p.splits; s0 += 8) {
+    float4 x[8], y[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      if (s0 + k < p.splits) {
+        x[k] = __ldcg(reinterpret_cast<const float4*>(sl + (size_t)(s0 + k) * sstride));
+        if (po) y[k] = __ldcg(reinterpret_cast<const float4*>(sl + (size_t)(s0 + k) * sstride + po));
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      if (s0 + k < p.splits) {
+        v[0] += x[k].x; v[1] += x[k].y; v[2] += x[k].z; v[3] += x[k].w;
+        if (po) {
+          vp[0] += y[k].x; vp[1] += y[k].y; vp[2] += y[k].z; vp[3] += y[k].w;
+        }
+      }
+    }
+  }
+  tc_apply4<EPI, SPLIT>(p, tile, j, c, v, vp, rs);
+}
+
 // ---------------------------------------------------------------------------
 // Epilogue of one unit by the four epilogue warps (128 threads).  Warp w reads
 // TMEM lanes 32*(w%4).. (rows of each M-tile) and writes the unit's
@@ -362,7 +405,7 @@ __device__ __forceinline__ void tc_apply4(const TcParams& p, int tile, int j, in
 // (tempty) right after.  The CTA that completes a tile (the last of its K
 // splits, or the only one) then applies the epilogue with all 128 threads over
 // (row, 4-column group) items, summing the splits' slots in split order
-// (deterministic).  Returns whether this CTA finished the tile.
+// (deterministic).  With p.defer every unit stops after staging its slot.
 // ---------------------------------------------------------------------------
 template <int EPI, bool SPLIT>
 __device__ __forceinline__ void tc_epilogue_unit(const TcParams& p, int u, int m, uint32_t tacc, uint64_t* tempty,
@@ -387,6 +430,7 @@ __device__ __forceinline__ void tc_epilogue_unit(const TcParams& p, int u, int m
   }
   ptx::tc_fence_before();
   if (lane == 0) ptx::mbar_arrive(tempty);
+  if (p.defer) return;   // gemm_fix_kernel sums the splits
   epi_bar();
   const int et = threadIdx.x & 127;
   if (et == 0) {
@@ -403,44 +447,11 @@ __device__ __forceinline__ void tc_epilogue_unit(const TcParams& p, int u, int m
   epi_bar();
   if (*last_flag) {
     __threadfence();
-    const int po = tc_partner_off<EPI>(p);
     const int ng = tc_groups<EPI>(p);
     const int items = m * ng;
-    const size_t sstride = (size_t)p.n_tiles * p.rows_max * p.bw;   // one split's slots
-    const float* base = p.ws + (size_t)tile * p.rows_max * p.bw;
-    // one item per thread per round; the partials of up to eight splits (and
-    // the residual) are loaded together, then summed in split order
-    for (int it = et; it < items; it += 128) {
-      const int j = it / ng, c = tc_group_col<EPI>(p, it - j * ng);
-      const float* sl = base + (size_t)j * p.bw + c;
-      float v[4] = {0.f, 0.f, 0.f, 0.f}, vp[4] = {0.f, 0.f, 0.f, 0.f}, rs[4] = {0.f, 0.f, 0.f, 0.f};
-      if (EPI == EPI_RESID) {
-        const int seq = p.rows ? p.rows[j] : j;
-        const int n0 = tile * p.bw + c;
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-          if (n0 + i < p.N) rs[i] = p.resid_src[(size_t)seq * p.N + n0 + i];
-      }
-      for (int s0 = 0; s0 < p.splits; s0 += 8) {
-        float4 x[8], y[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          if (s0 + k < p.splits) {
-            x[k] = __ldcg(reinterpret_cast<const float4*>(sl + (size_t)(s0 + k) * sstride));
-            if (po) y[k] = __ldcg(reinterpret_cast<const float4*>(sl + (size_t)(s0 + k) * sstride + po));
-          }
-        }
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          if (s0 + k < p.splits) {
-            v[0] += x[k].x; v[1] += x[k].y; v[2] += x[k].z; v[3] += x[k].w;
-            if (po) {
-              vp[0] += y[k].x; vp[1] += y[k].y; vp[2] += y[k].z; vp[3] += y[k].w;
-            }
-          }
-        }
-      }
-      tc_apply4<EPI, SPLIT>(p, tile, j, c, v, vp, rs);
+    for (int it = et; it < items; it += 128) {   // one item per thread per round
+      const int j = it / ng;
+      tc_fix_item<EPI, SPLIT>(p, tile, j, tc_group_col<EPI>(p, it - j * ng));
     }
   }
   epi_bar();

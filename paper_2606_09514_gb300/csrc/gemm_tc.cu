@@ -271,6 +271,29 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   if (warp == 1) ptx::tmem_dealloc(tmem_base, p.tmem_cols);
 }
 
+// Deferred fixup of a GEMM whose units only staged their partials: items
+// (tile, row, 4-column group) over the whole grid, each summing its splits in
+// split order (the same order, hence the same result, as the in-kernel
+// finisher) and applying the epilogue.  Consecutive threads take consecutive
+// column groups of a row, so the workspace reads are coalesced.
+template <int EPI, bool SPLIT>
+__global__ void __launch_bounds__(kTcFixThreads) gemm_fix_kernel(const TcParams p) {
+  pdl_wait();
+  pdl_trigger();
+  if (call_aborted(p.status)) return;
+  const int m = p.count ? *p.count : p.n;
+  if (m <= 0) return;
+  const int ng = tc_groups<EPI>(p);
+  const long long items = (long long)p.n_tiles * m * ng;
+  for (long long it = (long long)blockIdx.x * kTcFixThreads + threadIdx.x; it < items;
+       it += (long long)gridDim.x * kTcFixThreads) {
+    const int g = (int)(it % ng);
+    const long long r = it / ng;
+    const int j = (int)(r % m), tile = (int)(r / m);
+    tc_fix_item<EPI, SPLIT>(p, tile, j, tc_group_col<EPI>(p, g));
+  }
+}
+
 // ---------------------------------------------------------------------------
 // Host side
 // ---------------------------------------------------------------------------
@@ -430,6 +453,14 @@ int gemm_tc_prepare(Ctx& c) {
       if (c.tc_pstages[v] < 3) c.tc_panel = false;
     }
   }
+  // Above kTcDeferRows rows a tile's partials are too many for the one CTA
+  // that would finish it (m x 256 fp32 per split): a fixup kernel spreads
+  // them over all SMs.  BUDDY_TC_DEFER_ROWS overrides the threshold.
+  {
+    const char* env = getenv("BUDDY_TC_DEFER_ROWS");
+    const int thr = env && env[0] ? atoi(env) : kTcDeferRows;
+    c.tc_defer = c.maxB > thr;
+  }
   const char* lk_env = getenv("BUDDY_LAYER_KERNEL");
   c.use_lk = layer_kernel_supported(c) && lk_env && lk_env[0] == '1';   // opt-in
   if (c.use_lk && !c.lk_bar) {
@@ -451,7 +482,8 @@ int gemm_tc_prepare(Ctx& c) {
   return BUDDY_OK;
 }
 
-void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s) {
+// Kernel parameters of one GEMM call; *smem = its dynamic shared memory.
+static TcParams tc_params(const Ctx& c, const GemmArgs& a, size_t* smem_out) {
   const int which = a.which;
   TcParams p{};
   int N, K, tiles;
@@ -508,9 +540,18 @@ void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s) {
     smem = c.tc_psmem[v];
   }
   p.count_late = a.count_late ? 1 : 0;
+  p.defer = c.tc_defer ? 1 : 0;
   p.nq = c.nq;
   p.nkv = c.nkv;
   p.hd = c.hd;
+  *smem_out = smem;
+  return p;
+}
+
+void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s) {
+  const int which = a.which;
+  size_t smem = 0;
+  const TcParams p = tc_params(c, a, &smem);
   const CUtensorMap& tw = c.tmaps_host[(size_t)a.layer * 4 + which];
   const int xi = which == 0 || which == 2 ? 0 : (which == 1 ? 1 : 2);
   const CUtensorMap& tx = c.tmaps_host[(size_t)c.L * 4 + xi];
@@ -547,5 +588,27 @@ void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s) {
     }
   }
 }
+
+void launch_gemm_fix(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s) {
+  size_t smem = 0;
+  const TcParams p = tc_params(c, a, &smem);
+  const int fgrid = c.num_sms * (2048 / kTcFixThreads);
+  if (a.split) {
+    switch (epi) {
+      case EPI_QKV: launch_k(gemm_fix_kernel<EPI_QKV, true>, fgrid, kTcFixThreads, 0, s, c.pdl, p); break;
+      case EPI_STORE_F32: launch_k(gemm_fix_kernel<EPI_STORE_F32, true>, fgrid, kTcFixThreads, 0, s, c.pdl, p); break;
+      case EPI_RESID: launch_k(gemm_fix_kernel<EPI_RESID, true>, fgrid, kTcFixThreads, 0, s, c.pdl, p); break;
+      default: launch_k(gemm_fix_kernel<EPI_SWIGLU, true>, fgrid, kTcFixThreads, 0, s, c.pdl, p);
+    }
+  } else {
+    switch (epi) {
+      case EPI_QKV: launch_k(gemm_fix_kernel<EPI_QKV, false>, fgrid, kTcFixThreads, 0, s, c.pdl, p); break;
+      case EPI_STORE_F32: launch_k(gemm_fix_kernel<EPI_STORE_F32, false>, fgrid, kTcFixThreads, 0, s, c.pdl, p); break;
+      case EPI_RESID: launch_k(gemm_fix_kernel<EPI_RESID, false>, fgrid, kTcFixThreads, 0, s, c.pdl, p); break;
+      default: launch_k(gemm_fix_kernel<EPI_SWIGLU, false>, fgrid, kTcFixThreads, 0, s, c.pdl, p);
+    }
+  }
+}
+
 
 }  // namespace buddy

@@ -120,6 +120,7 @@ bool layer_kernel_supported(const Ctx& c);
 bool launch_layer_kernel(const Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, const float* src, float* H,
                          cudaStream_t s);
 void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s);
+void launch_gemm_fix(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s);   // with c.tc_defer
 
 struct Ctx {
   buddy_config cfg;
@@ -182,6 +183,9 @@ struct Ctx {
   bool tc_panel = false;
   int tc_panel_kb = 0, tc_pstages[2] = {1, 1}, tc_psmem[2] = {0, 0};
   uint32_t tc_panel_bytes[2] = {0, 0};
+  // deferred split-K fixup (batches above kTcDeferRows rows): a second kernel
+  // per GEMM sums the partials and applies the epilogue on every SM
+  bool tc_defer = false;
 
   // profiler: event pairs around kernel launches (direct-launch mode only)
   int profiling = 0;
