@@ -329,7 +329,7 @@ def run_ours(args, ws, rank, local):
     # the timed steps launch every middle layer (a layer no row selected exits
     # at once); the profiled steps launch only the selected ones
     per_layer = ("rmsnorm", "gemm_qkv", "qkv_finalize", "attention", "gemm_o", "gemm_gate_up", "gemm_down",
-                 "layer", "gemm_fixup")
+                 "layer", "gemm_fixup", "attn_merge")
     exec_layers = (prof.get("attention", (0, 0))[1] + prof.get("layer", (0, 0))[1]) / prof_steps
     per_layer_kernels = sum(prof.get(k, (0, 0))[1] for k in per_layer) / max(exec_layers * prof_steps, 1)
     graph_extra = max(s.n_layers - exec_layers, 0) * per_layer_kernels

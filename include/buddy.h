@@ -226,6 +226,7 @@ enum {
   BUDDY_PROF_ROUTE, BUDDY_PROF_COMPACT, BUDDY_PROF_OTHER,
   BUDDY_PROF_LAYER,   /* a whole block as one persistent kernel (small batches) */
   BUDDY_PROF_GEMM_FIXUP,   /* split-K sums + epilogues of the GEMMs (larger batches) */
+  BUDDY_PROF_ATTN_MERGE,   /* span merge of the tensor-core attention */
   BUDDY_PROF_NCLASS
 };
 

@@ -119,8 +119,7 @@ extern "C" int buddy_create(const buddy_config* cfg, buddy_ctx** out) {
   if ((e = cudaDeviceGetAttribute(&c.num_sms, cudaDevAttrMultiProcessorCount, c.device)) != cudaSuccess)
     return fail(e);
   const size_t B = c.maxB;
-  c.attn_chunk = attention_chunk();
-  c.attn_max_chunks = (c.max_pos + c.attn_chunk - 1) / c.attn_chunk;
+  c.attn_max_chunks = attention_max_spans(c.max_pos);
   const size_t hmax = (size_t)c.max_pos * (c.hd / 2);
   if ((e = dalloc(&c.rope_cos, hmax)) || (e = dalloc(&c.rope_sin, hmax)) ||
       (e = dalloc(&c.status, 4)) ||
@@ -130,7 +129,7 @@ extern "C" int buddy_create(const buddy_config* cfg, buddy_ctx** out) {
       (e = dalloc(&c.attn_m, B * c.nq * c.attn_max_chunks)) ||
       (e = dalloc(&c.attn_l, B * c.nq * c.attn_max_chunks)) ||
       (e = dalloc(&c.attn_acc, B * c.nq * c.attn_max_chunks * c.hd)) ||
-      (e = dalloc(&c.attn_ctr, B * c.nkv)) ||
+      (e = dalloc(&c.attn_ctr, B * c.nkv)) || (e = dalloc(&c.attn_meta, B + 2)) ||
       (e = dalloc(&c.dm_u, B * c.r)) || (e = dalloc(&c.mask, B * c.L)) ||
       (e = dalloc(&c.sel, B * c.Lm)) || (e = dalloc(&c.scores, B * c.Lm)) ||
       (e = dalloc(&c.rows, (size_t)c.L * B)) || (e = dalloc(&c.count, (size_t)c.L)) ||
@@ -254,7 +253,8 @@ extern "C" int buddy_set_profiling(buddy_ctx* ctx, int32_t on) {
 extern "C" const char* buddy_profile_class_name(int32_t cls) {
   static const char* names[BUDDY_PROF_NCLASS] = {"check", "rmsnorm", "gemm_qkv", "qkv_finalize",
                                                  "attention", "gemm_o", "gemm_gate_up", "gemm_down",
-                                                 "route", "compact", "other", "layer", "gemm_fixup"};
+                                                 "route", "compact", "other", "layer", "gemm_fixup",
+                                                 "attn_merge"};
   return (cls >= 0 && cls < BUDDY_PROF_NCLASS) ? names[cls] : "unknown";
 }
 
@@ -346,6 +346,10 @@ static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, c
   {
     ProfScope p(c, s, BUDDY_PROF_ATTENTION, 1, prof);
     launch_attention(c, sel, kv, l, c.q, c.attn_out, split ? c.attn_lo : nullptr, s);
+  }
+  if (attention_tc(c)) {
+    ProfScope p(c, s, BUDDY_PROF_ATTN_MERGE, 1, prof);
+    launch_attention_merge(c, sel, c.attn_out, split ? c.attn_lo : nullptr, s);
   }
   g = GemmArgs{};
   g.sel = sel; g.max_m = sel.n; g.split = split;

@@ -28,8 +28,15 @@ namespace buddy {
 template <int HD, bool SPLIT>
 __global__ void __launch_bounds__(kTcaThreads) attn_tc_kernel(AttnArgs<bf16> A) {
   extern __shared__ __align__(16) uint8_t smraw[];
-  __shared__ float sc[32];
+  __shared__ int sc[4];
   attn_tc_run<HD, SPLIT>(A, blockIdx.x, gridDim.x, smraw, sc, true);
+}
+
+template <int HD>
+__global__ void __launch_bounds__(kTcaMergeThreads) attn_tc_merge_kernel(AttnArgs<bf16> A) {
+  pdl_wait();
+  pdl_trigger();
+  attn_tc_merge_run<HD>(A);
 }
 
 // bf16 caches with at most 8 query heads per KV head: the tensor-core loop
@@ -37,14 +44,10 @@ template <int HD, bool SPLIT>
 static void attn_tc_impl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q, void* out,
                          void* out_lo, cudaStream_t s) {
   const size_t smem = attn_tc_smem_bytes(HD, c.maxB);
-  static bool attr_set = false;   // one per instantiation
-  static int occ = 0;
+  static int occ = 0;   // one per instantiation
   static size_t occ_smem = 0;
-  if (!attr_set) {
-    cudaFuncSetAttribute(attn_tc_kernel<HD, SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    attr_set = true;
-  }
   if (occ == 0 || occ_smem != smem) {
+    cudaFuncSetAttribute(attn_tc_kernel<HD, SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, attn_tc_kernel<HD, SPLIT>, kTcaThreads, smem) !=
         cudaSuccess)
       occ = 1;
@@ -53,8 +56,16 @@ static void attn_tc_impl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int
   const int grid = c.num_sms * std::max(1, std::min(occ, 4));
   AttnArgs<bf16> A{q, sel.rows, sel.count, sel.n, c.nq, c.nkv, kv.len, kv.seq_off, kv.cap,
                    (const bf16*)kv.k_cache[layer], (const bf16*)kv.v_cache[layer], c.attn_max_chunks, c.attn_m,
-                   c.attn_l, c.attn_acc, c.attn_ctr, (bf16*)out, (bf16*)out_lo, c.status};
+                   c.attn_l, c.attn_acc, c.attn_ctr, (bf16*)out, (bf16*)out_lo, c.status, c.attn_meta};
   launch_k(attn_tc_kernel<HD, SPLIT>, grid, kTcaThreads, smem, s, c.pdl, A);
+}
+
+template <int HD>
+static void attn_tc_merge_impl(const Ctx& c, RowSel sel, void* out, void* out_lo, cudaStream_t s) {
+  AttnArgs<bf16> A{nullptr, sel.rows, sel.count, sel.n, c.nq, c.nkv, nullptr, nullptr, nullptr, nullptr, nullptr,
+                   c.attn_max_chunks, c.attn_m, c.attn_l, c.attn_acc, nullptr, (bf16*)out, (bf16*)out_lo,
+                   c.status, c.attn_meta};
+  launch_k(attn_tc_merge_kernel<HD>, c.maxB * c.nkv, kTcaMergeThreads, 0, s, c.pdl, A);
 }
 
 template <typename T, int HD, int GP>
@@ -100,13 +111,28 @@ static void attn_group(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int l
   }
 }
 
-// Spans are at least one chunk long, so the partial buffers hold
-// ceil(max_pos / kChunk) spans per (row, head).
-int attention_chunk() { return kChunk; }
+// Partial slots per (row, query head): the CUDA-core loop's spans are at least
+// kChunk positions long; the tensor-core loop's at least kTcaMinShare, plus
+// one for a share boundary.
+int attention_max_spans(int max_pos) {
+  return std::max((max_pos + kChunk - 1) / kChunk, attn_tc_max_spans(max_pos));
+}
+
+// bf16 caches with at most 8 query heads per KV head whose per-row tables fit
+// next to the chunk buffers take the tensor-core loop (and its merge kernel)
+bool attention_tc(const Ctx& c) {
+  return c.dtype == BUDDY_DTYPE_BF16 && c.nq / c.nkv <= 8 &&
+         attn_tc_smem_bytes(c.hd, c.maxB) <= (size_t)kTcaSmemLimit;
+}
+
+void launch_attention_merge(const Ctx& c, RowSel sel, void* out, void* out_lo, cudaStream_t s) {
+  if (c.hd == 128) attn_tc_merge_impl<128>(c, sel, out, out_lo, s);
+  else attn_tc_merge_impl<64>(c, sel, out, out_lo, s);
+}
 
 void launch_attention(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q,
                       void* out, void* out_lo, cudaStream_t s) {
-  if (c.dtype == BUDDY_DTYPE_BF16 && c.nq / c.nkv <= 8) {
+  if (attention_tc(c)) {
     if (c.hd == 128) {
       if (out_lo) attn_tc_impl<128, true>(c, sel, kv, layer, q, out, out_lo, s);
       else attn_tc_impl<128, false>(c, sel, kv, layer, q, out, out_lo, s);

@@ -81,6 +81,7 @@ struct AttnArgs {
   T* out;
   T* out_lo;
   const int32_t* status;
+  int32_t* meta;   // tensor-core loop: row prefix and share for its merge kernel
 };
 
 // Dynamic shared memory used by attn_run (bytes): double-buffered K (rows
@@ -105,8 +106,10 @@ inline size_t attn_smem_bytes(size_t fixed, int G, int hd, int max_spans, int ma
 // a), loading D of their spans' partials at a time; the tpo results are then
 // combined by a lane butterfly (every thread ends with the same values).  When
 // the outputs outnumber the threads, the threads take them in rounds of NT.
-template <typename T, int HD, int NT>
+// B2: the partial maxima are base-2 logarithms (weights 2^(m - M)).
+template <typename T, int HD, int NT, bool B2 = false>
 __device__ __forceinline__ void attn_span_merge(const AttnArgs<T>& A, int j, int g, int nsp, size_t obase, int tid) {
+  auto ex = [](float x) { return B2 ? exp2f(x) : expf(x); };
   constexpr int D = NT >= 256 ? 16 : 8;   // partials in flight per thread
   const int nq = A.nq, G = A.nq / A.nkv, max_spans = A.max_spans;
   const float* __restrict__ part_acc = A.part_acc;
@@ -145,7 +148,7 @@ __device__ __forceinline__ void attn_span_merge(const AttnArgs<T>& A, int j, int
       for (int k = 0; k < D; ++k) {
         if (c0 + k * tpo < nsp) {
           const float mn = fmaxf(M, ms[k]);
-          const float fo = expf(M - mn), fn = expf(ms[k] - mn);
+          const float fo = ex(M - mn), fn = ex(ms[k] - mn);
           a.x = a.x * fo + t[k].x * fn;
           a.y = a.y * fo + t[k].y * fn;
           a.z = a.z * fo + t[k].z * fn;
@@ -160,7 +163,7 @@ __device__ __forceinline__ void attn_span_merge(const AttnArgs<T>& A, int j, int
       const float ax = __shfl_xor_sync(0xffffffffu, a.x, o), ay = __shfl_xor_sync(0xffffffffu, a.y, o);
       const float az = __shfl_xor_sync(0xffffffffu, a.z, o), aw = __shfl_xor_sync(0xffffffffu, a.w, o);
       const float mn = fmaxf(M, M2);
-      const float f1 = M == -INFINITY ? 0.f : expf(M - mn), f2 = M2 == -INFINITY ? 0.f : expf(M2 - mn);
+      const float f1 = M == -INFINITY ? 0.f : ex(M - mn), f2 = M2 == -INFINITY ? 0.f : ex(M2 - mn);
       a.x = a.x * f1 + ax * f2;
       a.y = a.y * f1 + ay * f2;
       a.z = a.z * f1 + az * f2;

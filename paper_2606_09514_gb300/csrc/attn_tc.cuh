@@ -1,23 +1,40 @@
 // Decode attention on the tensor cores (bf16 caches, head dim 64 or 128, at
-// most 8 query heads per KV head).  Same work decomposition and results as the
-// SIMT work loop in attn_common.cuh (items = row x KV head x span of P
-// positions, split spans merged in span order by the last CTA to finish), but
-// inside a span each of the four warps streams its own 32-position chunks:
+// most 8 query heads per KV head), Eq. 9 for every active row and KV head.
 //
-//   * K and V rows of the chunk are copied with 16-byte cp.async into the
-//     warp's double buffer (rows padded by 16 bytes: ldmatrix conflict-free);
-//   * logits S = Q K^T with mma.sync m16n8k16 (bf16 in, fp32 accumulate): the
-//     query heads are the 16 rows of A (heads >= G are zero), K rows feed B
-//     through ldmatrix;
-//   * online softmax on the accumulator fragments (quad shuffles per row);
-//   * O += P V with the probabilities taken straight from the S fragments as
-//     the A operand and V through ldmatrix.trans.
+// Work decomposition: the (row j, KV head g) streams of positions 0..len[i]
+// are laid end to end (row-major, heads inside a row) and every warp of the
+// grid takes an equal contiguous share of that sequence (a multiple of the
+// chunk, at least two chunks).  A share may end in the middle of a stream and
+// cover several short ones; the piece of a stream that one warp holds is a
+// span.  A stream held by one warp is written out directly; otherwise every
+// warp writes its span's partial (running max, sum of exponentials,
+// unnormalised output), and the partials are merged in span order
+// (deterministic): for at most kTcaWarpMerge spans by the warp that completes
+// the stream last (an arrival counter per stream), for more (small batches,
+// long rows) by attn_tc_merge_kernel, launched right after, one CTA per
+// stream.  Because warps never wait for each other, each streams its share
+// without a break: the copies of the next span are in flight while the
+// current one finishes (or merges).
+//
+// Inside a share a warp walks chunks of up to kTcaChunk positions (never
+// crossing a stream end):
+//
+//   * K and V rows of the chunk are copied with 16-byte cp.async into one of
+//     the warp's kTcaStages buffers (rows padded by 16 bytes: ldmatrix
+//     conflict-free); kTcaStages - 1 chunks are in flight while one is used;
+//   * logits, transposed: S^T = K Q^T with mma.sync m16n8k16 (bf16 in, fp32
+//     accumulate): 16 positions are the rows of A (K rows through ldmatrix),
+//     the query heads the 8 columns of B (heads >= G are zero);
+//   * online softmax per head (a column) on the accumulator fragments, in
+//     base 2 (the queries carry log2(e) / sqrt(d_h));
+//   * O^T += V^T P^T: 16 channels are the rows of A (V through
+//     ldmatrix.trans), the probabilities, transposed in registers
+//     (movmatrix), the B operand.
 //
 // With SPLIT (the first block, which feeds the router) the scaled queries and
 // the probabilities are each given as bf16 hi + lo and every product is issued
 // for both terms, so the contractions carry ~16 mantissa bits; otherwise one
-// bf16 term each.  The four warps' running (max, sum, output) are combined in
-// shared memory.
+// bf16 term each.
 #pragma once
 
 #include <cuda_runtime.h>
@@ -27,19 +44,36 @@
 
 namespace buddy {
 
-constexpr int kTcaChunk = 32;     // positions per warp chunk
-constexpr int kTcaWarps = 4;
+#ifndef BUDDY_TCA_CHUNK
+#define BUDDY_TCA_CHUNK 32
+#endif
+constexpr int kTcaChunk = BUDDY_TCA_CHUNK;   // positions per warp chunk (16 or 32)
+#ifndef BUDDY_TCA_WARPS
+#define BUDDY_TCA_WARPS 4
+#endif
+constexpr int kTcaWarps = BUDDY_TCA_WARPS;
 constexpr int kTcaThreads = 32 * kTcaWarps;
+#ifndef BUDDY_TCA_STAGES
+#define BUDDY_TCA_STAGES 3
+#endif
+constexpr int kTcaStages = BUDDY_TCA_STAGES;   // chunk buffers per warp (kTcaStages - 1 in flight)
+constexpr int kTcaMinShare = 2 * kTcaChunk;   // positions of a warp's share, at least
+constexpr int kTcaMergeThreads = 256;         // merge kernel: one CTA per stream
+constexpr int kTcaWarpMerge = 4;              // streams of at most this many spans merge in the kernel
 
 template <int HD>
 __host__ __device__ constexpr size_t attn_tc_smem_fixed() {
-  // per warp: two buffers of K and V rows, each row padded by 8 bf16
-  return (size_t)kTcaWarps * 2 * 2 * kTcaChunk * (HD + 8) * 2;
+  // per warp: kTcaStages buffers of K and V rows, each row padded by 8 bf16
+  return (size_t)kTcaWarps * kTcaStages * 2 * kTcaChunk * (HD + 8) * 2;
 }
+constexpr int kTcaSmemLimit = 226 * 1024;   // dynamic shared memory of one CTA (227 KiB less static)
 inline size_t attn_tc_smem_bytes(int hd, int max_rows) {
   const size_t fixed = hd == 128 ? attn_tc_smem_fixed<128>() : attn_tc_smem_fixed<64>();
   return fixed + (size_t)(max_rows + 1) * 4 + 8 + (size_t)max_rows * 16;
 }
+// Spans one stream of at most max_pos positions can be cut into: shares are at
+// least kTcaMinShare positions, and the first and last may be partial.
+inline int attn_tc_max_spans(int max_pos) { return (max_pos + kTcaMinShare - 1) / kTcaMinShare + 1; }
 
 namespace tca {
 
@@ -63,26 +97,106 @@ __device__ __forceinline__ void ldsm_x4_t(const void* p, uint32_t& r0, uint32_t&
                : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
                : "r"((uint32_t)__cvta_generic_to_shared(p)));
 }
-// D (16x8 fp32) += A (16x16 bf16, rows 8..15 zero) * B (16x8 bf16).  Only
-// rows 0..7 are kept (d0, d1 of this thread); rows 8..15 go to scratch z.
-__device__ __forceinline__ void mma16816(float& d0, float& d1, float (&z)[2], uint32_t a0, uint32_t a2, uint32_t b0,
-                                         uint32_t b1) {
+// D (16x8 fp32) += A (16x16 bf16) * B (16x8 bf16)
+__device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
   asm volatile(
       "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
       "{%0,%1,%2,%3};"
-      : "+f"(d0), "+f"(d1), "+f"(z[0]), "+f"(z[1])
-      : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+// transpose of an 8x8 b16 matrix held one 32-bit pair per thread
+__device__ __forceinline__ uint32_t movt(uint32_t x) {
+  uint32_t y;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+  return y;
+}
+// 2^x (hardware approximation, relative error ~2^-22; 2^-inf = 0)
+__device__ __forceinline__ float exp2a(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
 }  // namespace tca
 
-// Processes this CTA's share of one layer's attention (kTcaThreads threads).
-// Smem layout: per-warp K/V double buffers, then the row prefix and the rows'
-// cache offsets, positions and head strides.  `sc` is 32 floats of scratch.
+// Merge of a (row j, KV head g)'s nsp <= kTcaWarpMerge span partials by one
+// warp: lane -> (head, four channels) per round of 32 lanes; two rounds'
+// partials (every span's output, max and sum) are loaded at once, then each
+// output is sum_s 2^(m_s - M) o_s / sum_s 2^(m_s - M) l_s, in span order.
+template <int HD>
+__device__ __forceinline__ void attn_tc_warp_merge(const AttnArgs<bf16>& A, int j, int g, int nsp, size_t obase,
+                                                   int lane) {
+  constexpr int Q = HD / 4;      // float4 outputs per head
+  constexpr int HPR = 32 / Q;    // heads per round (1 or 2)
+  constexpr int NS = kTcaWarpMerge;
+  const int G = A.nq / A.nkv, ms = A.max_spans;
+  const size_t hb0 = ((size_t)j * A.nq + (size_t)g * G) * ms;
+  const int hsub = lane / Q, e0 = (lane % Q) * 4;
+  for (int r0 = 0; r0 * HPR < G; r0 += 2) {
+    float4 v[2][NS];
+    float mv[2][NS], lv[2][NS];
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int h = (r0 + u) * HPR + hsub;
+#pragma unroll
+      for (int s = 0; s < NS; ++s) {
+        if (h < G && s < nsp) {
+          const size_t slot = hb0 + (size_t)h * ms + s;
+          v[u][s] = __ldcg(reinterpret_cast<const float4*>(A.part_acc + slot * HD + e0));
+          mv[u][s] = __ldcg(A.part_m + slot);
+          lv[u][s] = __ldcg(A.part_l + slot);
+        }
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int h = (r0 + u) * HPR + hsub;
+      if (h >= G) continue;
+      float M = mv[u][0];
+#pragma unroll
+      for (int s = 1; s < NS; ++s)
+        if (s < nsp) M = fmaxf(M, mv[u][s]);
+      float L = 0.f;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int s = 0; s < NS; ++s) {
+        if (s < nsp) {
+          const float w = tca::exp2a(mv[u][s] - M);
+          L += w * lv[u][s];
+          acc.x += w * v[u][s].x;
+          acc.y += w * v[u][s].y;
+          acc.z += w * v[u][s].z;
+          acc.w += w * v[u][s].w;
+        }
+      }
+      const float inv = 1.f / L;
+      const size_t o = obase + (size_t)h * HD + e0;
+      store_out(A.out, A.out_lo, o + 0, acc.x * inv);
+      store_out(A.out, A.out_lo, o + 1, acc.y * inv);
+      store_out(A.out, A.out_lo, o + 2, acc.z * inv);
+      store_out(A.out, A.out_lo, o + 3, acc.w * inv);
+    }
+  }
+}
+
+// Position in the sequence of streams: row j (index into the active rows), KV
+// head g, position p of that stream (np = the stream's length).
+struct TcaCursor {
+  int j, g, p, np;
+};
+
+// Processes warp `gw` of `nw` warps' share of one layer's attention.  Smem:
+// per-warp K/V buffers, then the row prefix (stream starts of each row, in
+// positions) and the rows' cache offsets, lengths and head strides, written by
+// warp 0 of every CTA before the CTA-wide barrier.
 template <int HD, bool SPLIT>
-__device__ __forceinline__ void attn_tc_run(const AttnArgs<bf16>& A, int cta, int ncta, uint8_t* smem, float* sc,
+__device__ __forceinline__ void attn_tc_run(const AttnArgs<bf16>& A, int cta, int ncta, uint8_t* smem, int* sc,
                                             bool pdl) {
   static_assert(HD == 64 || HD == 128, "HD");
+  static_assert(kTcaChunk == 16 || kTcaChunk == 32, "chunk");
+  constexpr int CH = kTcaChunk, NST = kTcaStages;
   constexpr int KROW = HD + 8;                    // padded row (elements)
   constexpr int KSTEPS = HD / 16;                 // k-steps of the logits
   constexpr int DT = HD / 8;                      // output n-tiles
@@ -96,124 +210,171 @@ __device__ __forceinline__ void attn_tc_run(const AttnArgs<bf16>& A, int cta, in
     if (pdl) pdl_wait();
     return;
   }
-  bf16* wbuf = reinterpret_cast<bf16*>(smem) + (size_t)warp * 2 * 2 * kTcaChunk * KROW;   // this warp's buffers
+  bf16* wbuf = reinterpret_cast<bf16*>(smem) + (size_t)warp * NST * 2 * CH * KROW;   // this warp's buffers
   int* pref = reinterpret_cast<int*>(smem + attn_tc_smem_fixed<HD>());
   int64_t* rbase = reinterpret_cast<int64_t*>((reinterpret_cast<uintptr_t>(pref + m + 1) + 7) & ~uintptr_t(7));
   int* rnp = reinterpret_cast<int*>(rbase + m);
   int* rhs = rnp + m;
-  float* mw = reinterpret_cast<float*>(smem);                   // merge: [warps][8] max
-  float* lw = mw + kTcaWarps * 8;                               //        [warps][8] sum
-  float* ow = lw + kTcaWarps * 8;                               //        [warps][8][HD] output
-  int* last_s_p = reinterpret_cast<int*>(sc + 24);
-  int* span_s_p = reinterpret_cast<int*>(sc + 25);
 
-  // positions per row and their total -> span length P (as attn_run)
+  // streams per row (nkv of length len + 1) and their prefix; the share
   if (warp == 0) {
-    long long tot = 0;
-    for (int j = lane; j < m; j += 32) {
-      const int i = rows ? rows[j] : j;
-      const int np = A.len[i] + 1;
-      rnp[j] = np;
-      rbase[j] = A.seq_off[i] * nkv * HD;
-      rhs[j] = A.cap[i] * HD;
-      pref[j + 1] = np;
-      tot += np;
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
-    __syncwarp();
-    // about one item per CTA; a span is a multiple of the four warps' chunks
-    const long long want = (tot * nkv + ncta - 1) / ncta;
-    constexpr int kQ = kTcaChunk * kTcaWarps;
-    const int P0 = (int)min((long long)kMaxSpan, max((long long)kQ, want));
-    const int P = (P0 + kQ - 1) / kQ * kQ;
     int carry = 0;
     for (int b = 0; b < m; b += 32) {
       const int j = b + lane;
-      int ns = 0;
-      if (j < m) ns = (pref[j + 1] + P - 1) / P;
-      int x = ns;
+      int x = 0;
+      if (j < m) {
+        const int i = rows ? rows[j] : j;
+        const int np = A.len[i] + 1;
+        rnp[j] = np;
+        rbase[j] = A.seq_off[i] * nkv * HD;
+        rhs[j] = A.cap[i] * HD;
+        x = np * nkv;
+      }
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
         const int y = __shfl_up_sync(0xffffffffu, x, o);
         if (lane >= o) x += y;
       }
-      __syncwarp();
       if (j < m) pref[j + 1] = carry + x;
       carry += __shfl_sync(0xffffffffu, x, 31);
     }
     if (lane == 0) {
       pref[0] = 0;
-      *span_s_p = P;
+      const int nw = ncta * kTcaWarps;
+      const int even = (carry + nw - 1) / nw;
+      sc[0] = max(kTcaMinShare, (even + CH - 1) / CH * CH);
+    }
+    // the merge kernel's copy of the prefix and the share
+    if (cta == 0) {
+      __syncwarp();
+      for (int j = lane; j < m; j += 32) A.meta[j + 1] = pref[j + 1];
+      if (lane == 0) {
+        A.meta[0] = 0;
+        A.meta[m + 1] = sc[0];
+      }
     }
   }
   __syncthreads();
-  const int P = *span_s_p;
-  const int total = pref[m] * nkv;
-  const float scale = rsqrtf((float)HD);
-  bool waited = !pdl;
-  const int h0 = lane >> 2, c2 = (lane & 3) * 2;   // fragment row (head) and column pair
+  const int share = sc[0];
+  const int total = pref[m];
+  const int gw = cta * kTcaWarps + warp;
+  const long long a0 = (long long)gw * share;
+  if (a0 >= total) {   // nothing for this warp
+    if (pdl) {
+      pdl_wait();
+      pdl_trigger();
+    }
+    return;
+  }
+  const int a = (int)a0, b = min(total, a + share);
 
-  for (int item = cta; item < total; item += ncta) {
-    const int g = item % nkv;
-    const int js = item / nkv;
+  // cursor at flattened position x (binary search of the row prefix)
+  auto seek = [&](int x) {
     int lo = 0, hi = m;
     while (hi - lo > 1) {
       const int mid = (lo + hi) >> 1;
-      if (pref[mid] <= js) lo = mid;
+      if (pref[mid] <= x) lo = mid;
       else hi = mid;
     }
-    const int j = lo, sp = js - pref[j];
-    const int npos = rnp[j];
-    const int nsp = pref[j + 1] - pref[j];
-    const int s0 = sp * P, s1 = min(npos, s0 + P);
-    const int nch = (s1 - s0 + kTcaChunk - 1) / kTcaChunk;   // chunks of the span
-    const int64_t kvo = rbase[j] + (int64_t)g * rhs[j];
-    const bf16* Kbase = A.Kc + kvo;
-    const bf16* Vbase = A.Vc + kvo;
-
-    // this warp's chunks: c = warp, warp + 4, ...
-    auto issue = [&](int c, int buf) {
-      const int p0 = s0 + c * kTcaChunk, cnt = min(kTcaChunk, s1 - p0);
-      bf16* Kd = wbuf + (size_t)buf * 2 * kTcaChunk * KROW;
-      bf16* Vd = Kd + kTcaChunk * KROW;
-      for (int x = lane; x < cnt * V16; x += 32) {
-        const int p = x / V16, s = x - p * V16;
-        cp_async16(Kd + p * KROW + s * 8, Kbase + (size_t)(p0 + p) * HD + s * 8);
-        cp_async16(Vd + p * KROW + s * 8, Vbase + (size_t)(p0 + p) * HD + s * 8);
+    TcaCursor c;
+    c.j = lo;
+    c.np = rnp[lo];
+    const int off = x - pref[lo];
+    c.g = off / c.np;
+    c.p = off - c.g * c.np;
+    return c;
+  };
+  // positions of the chunk at cursor c (flattened position x)
+  auto chunk_len = [&](const TcaCursor& c, int x) { return min(CH, min(c.np - c.p, b - x)); };
+  // advance past a chunk of n positions (never beyond the stream end)
+  auto advance = [&](TcaCursor& c, int n) {
+    c.p += n;
+    if (c.p == c.np) {
+      c.p = 0;
+      if (++c.g == nkv) {
+        c.g = 0;
+        if (++c.j < m) c.np = rnp[c.j];
       }
-      // rows past the span end: zero V (their probabilities are 0, and 0 times
-      // stale shared memory could be NaN); K is masked on the logits
-      for (int x = cnt * V16 + lane; x < kTcaChunk * V16; x += 32) {
-        const int p = x / V16, s = x - p * V16;
-        *reinterpret_cast<uint4*>(Vd + p * KROW + s * 8) = make_uint4(0u, 0u, 0u, 0u);
-      }
-      cp_async_commit();
-    };
-    const int c_first = warp;
-    const bool has_work = c_first < nch;
-    if (!waited) {
-      // a chunk without the new token (position npos - 1) may be copied first
-      const bool has_new = has_work && s0 + (c_first + 1) * kTcaChunk >= npos;
-      if (has_work && !has_new) issue(c_first, 0);
-      pdl_wait();
-      pdl_trigger();
-      waited = true;
-      if (has_work && has_new) issue(c_first, 0);
-    } else if (has_work) {
-      issue(c_first, 0);
     }
-    // query fragments: rows = heads (h0 < G), columns = dims; scaled
-    uint32_t qh[KSTEPS][2], ql[KSTEPS][2];
-    {
-      const float* qj = A.q + (size_t)j * nq * HD + (size_t)g * G * HD + (size_t)h0 * HD;
+  };
+  auto issue = [&](const TcaCursor& c, int cnt, int buf) {
+    const int64_t kvo = rbase[c.j] + (int64_t)c.g * rhs[c.j] + (int64_t)c.p * HD;
+    bf16* Kd = wbuf + (size_t)buf * 2 * CH * KROW;
+    bf16* Vd = Kd + CH * KROW;
+    // lane -> (row lane / V16 + RPI * i, 16-byte piece lane % V16)
+    constexpr int RPI = 32 / V16;
+    const int pl = lane / V16, sl = lane % V16;
+    const bf16* ks = A.Kc + kvo + pl * HD + sl * 8;
+    const bf16* vs = A.Vc + kvo + pl * HD + sl * 8;
+    const int so = pl * KROW + sl * 8;
+#pragma unroll 4
+    for (int r = 0; r + pl < cnt; r += RPI) {
+      cp_async16(Kd + so + r * KROW, ks + (size_t)r * HD);
+      cp_async16(Vd + so + r * KROW, vs + (size_t)r * HD);
+    }
+    // rows past the chunk end: zero V (their probabilities are 0, and 0 times
+    // stale shared memory could be NaN); K is masked on the logits
+    for (int x = cnt * V16 + lane; x < CH * V16; x += 32) {
+      const int r = x / V16, q = x - r * V16;
+      *reinterpret_cast<uint4*>(Vd + r * KROW + q * 8) = make_uint4(0u, 0u, 0u, 0u);
+    }
+  };
+
+  // prologue: kTcaStages - 1 chunks in flight (one commit group each, empty
+  // past the share); chunks without the new token (the last position of a
+  // stream, written by the preceding kernel) may be copied before the wait
+  TcaCursor ci = seek(a);
+  int xi = a;
+  int k0 = 0;
+  if (pdl) {
+    for (; k0 < NST - 1 && xi < b; ++k0) {
+      const int cnt = chunk_len(ci, xi);
+      if (ci.p + cnt == ci.np) break;
+      issue(ci, cnt, k0);
+      cp_async_commit();
+      advance(ci, cnt);
+      xi += cnt;
+    }
+    pdl_wait();
+    pdl_trigger();
+  }
+  for (int k = k0; k < NST - 1; ++k) {
+    if (xi < b) {
+      const int cnt = chunk_len(ci, xi);
+      issue(ci, cnt, k);
+      advance(ci, cnt);
+      xi += cnt;
+    }
+    cp_async_commit();
+  }
+
+  const float scale = 1.4426950408889634f * rsqrtf((float)HD);   // log2(e) / sqrt(d_h)
+  const int h0 = lane >> 2, c2 = (lane & 3) * 2;   // fragment row (head) and column pair
+  TcaCursor cc = seek(a);
+  int xc = a;
+  uint32_t qh[KSTEPS][2], ql[KSTEPS][2];
+  float mrun[2], lrun[2];   // heads c2, c2 + 1
+  float o[DT / 2][4];       // O^T: channels 16 * t + lane / 4 (+8) x heads c2, c2 + 1
+  for (int k = 0; xc < b; ++k) {
+    if (xi < b) {
+      const int cnt = chunk_len(ci, xi);
+      issue(ci, cnt, (k + NST - 1) % NST);
+      advance(ci, cnt);
+      xi += cnt;
+    }
+    cp_async_commit();
+    const int cnt = chunk_len(cc, xc);
+    if (xc == a || cc.p == 0) {
+      // a new span: query fragments as the B operand (column = head h0 < G,
+      // rows = dims), scaled by log2(e) / sqrt(d_h), and a fresh running state
+      const float* qj = A.q + ((size_t)cc.j * nq + (size_t)cc.g * G + h0) * HD;
 #pragma unroll
       for (int kk = 0; kk < KSTEPS; ++kk) {
         float x0 = 0.f, x1 = 0.f, x2 = 0.f, x3 = 0.f;
         if (h0 < G) {
-          const float2 a = *reinterpret_cast<const float2*>(qj + kk * 16 + c2);
-          const float2 b = *reinterpret_cast<const float2*>(qj + kk * 16 + 8 + c2);
-          x0 = a.x * scale; x1 = a.y * scale; x2 = b.x * scale; x3 = b.y * scale;
+          const float2 u = *reinterpret_cast<const float2*>(qj + kk * 16 + c2);
+          const float2 v = *reinterpret_cast<const float2*>(qj + kk * 16 + 8 + c2);
+          x0 = u.x * scale; x1 = u.y * scale; x2 = v.x * scale; x3 = v.y * scale;
         }
         if (SPLIT) {
           tca::split_pack(x0, x1, qh[kk][0], ql[kk][0]);
@@ -223,154 +384,184 @@ __device__ __forceinline__ void attn_tc_run(const AttnArgs<bf16>& A, int cta, in
           qh[kk][1] = tca::pack_bf16(x2, x3);
         }
       }
-    }
-    float mrun = -INFINITY, lrun = 0.f;
-    float o[DT][2];
-    float z[2] = {0.f, 0.f};   // rows 8..15 of every product (padding heads)
+      mrun[0] = mrun[1] = -INFINITY;
+      lrun[0] = lrun[1] = 0.f;
 #pragma unroll
-    for (int t = 0; t < DT; ++t) o[t][0] = o[t][1] = 0.f;
+      for (int t = 0; t < DT / 2; ++t) o[t][0] = o[t][1] = o[t][2] = o[t][3] = 0.f;
+    }
+    cp_async_wait<NST - 1>();
+    __syncwarp();
+    const bf16* Ks = wbuf + (size_t)(k % NST) * 2 * CH * KROW;
+    const bf16* Vs = Ks + CH * KROW;
+    // S^T for MT tiles of 16 positions: two accumulators per tile (even and
+    // odd k-steps) for independent MMA chains
+    constexpr int MT = CH / 16;
+    float sv[MT][4];
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) {
+      float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+      // lanes 0-7 / 8-15: positions 16*mt + 0..7 / 8..15 of dims 16kk + 0..7;
+      // lanes 16-31: the same positions, dims 16kk + 8..15
+      const bf16* kr = Ks + (size_t)(mt * 16 + (lane & 7) + 8 * ((lane >> 3) & 1)) * KROW + 8 * (lane >> 4);
+#pragma unroll
+      for (int kk = 0; kk < KSTEPS; ++kk) {
+        uint32_t a0, a1, a2, a3;
+        tca::ldsm_x4(kr + kk * 16, a0, a1, a2, a3);
+        tca::mma16816(acc[kk & 1], a0, a1, a2, a3, qh[kk][0], qh[kk][1]);
+        if (SPLIT) tca::mma16816(acc[kk & 1], a0, a1, a2, a3, ql[kk][0], ql[kk][1]);
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) sv[mt][i] = acc[0][i] + acc[1][i];
+    }
+    // online softmax per head: this lane holds positions 16*mt + lane/4 (+8)
+    // of heads c2 (elements 0, 2) and c2 + 1 (elements 1, 3)
+    float cm[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) {
+      const int p0 = mt * 16 + h0;
+      if (p0 >= cnt) sv[mt][0] = sv[mt][1] = -INFINITY;
+      if (p0 + 8 >= cnt) sv[mt][2] = sv[mt][3] = -INFINITY;
+      cm[0] = fmaxf(cm[0], fmaxf(sv[mt][0], sv[mt][2]));
+      cm[1] = fmaxf(cm[1], fmaxf(sv[mt][1], sv[mt][3]));
+    }
+    float alpha[2], ps[2];
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+#pragma unroll
+      for (int off = 4; off < 32; off <<= 1) cm[e] = fmaxf(cm[e], __shfl_xor_sync(0xffffffffu, cm[e], off));
+      const float mn = fmaxf(mrun[e], cm[e]);
+      alpha[e] = tca::exp2a(mrun[e] - mn);   // 0 while mrun is -inf
+      mrun[e] = mn;
+      ps[e] = 0.f;
+    }
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        sv[mt][i] = tca::exp2a(sv[mt][i] - mrun[i & 1]);
+        ps[i & 1] += sv[mt][i];
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+#pragma unroll
+      for (int off = 4; off < 32; off <<= 1) ps[e] += __shfl_xor_sync(0xffffffffu, ps[e], off);
+      lrun[e] = lrun[e] * alpha[e] + ps[e];
+    }
+#pragma unroll
+    for (int t = 0; t < DT / 2; ++t) {
+      o[t][0] *= alpha[0];
+      o[t][1] *= alpha[1];
+      o[t][2] *= alpha[0];
+      o[t][3] *= alpha[1];
+    }
+    // O^T += V^T P^T, one k-step per tile of 16 positions
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) {
+      // P^T as B: transpose of the (positions x heads) fragments
+      uint32_t bh0, bh1, bl0 = 0, bl1 = 0;
+      if (SPLIT) {
+        uint32_t x0, y0, x1, y1;
+        tca::split_pack(sv[mt][0], sv[mt][1], x0, y0);
+        tca::split_pack(sv[mt][2], sv[mt][3], x1, y1);
+        bh0 = tca::movt(x0);
+        bh1 = tca::movt(x1);
+        bl0 = tca::movt(y0);
+        bl1 = tca::movt(y1);
+      } else {
+        bh0 = tca::movt(tca::pack_bf16(sv[mt][0], sv[mt][1]));
+        bh1 = tca::movt(tca::pack_bf16(sv[mt][2], sv[mt][3]));
+      }
+      // ldmatrix.trans groups: lanes 0-7 / 8-15 / 16-23 / 24-31 address
+      // positions 0..7 / 0..7 / 8..15 / 8..15 at channels +0 / +8 / +0 / +8
+      const bf16* vr = Vs + (size_t)(mt * 16 + (lane & 7) + 8 * (lane >> 4)) * KROW + 8 * ((lane >> 3) & 1);
+#pragma unroll
+      for (int t = 0; t < DT / 2; ++t) {
+        uint32_t a0, a1, a2, a3;
+        tca::ldsm_x4_t(vr + t * 16, a0, a1, a2, a3);
+        tca::mma16816(o[t], a0, a1, a2, a3, bh0, bh1);
+        if (SPLIT) tca::mma16816(o[t], a0, a1, a2, a3, bl0, bl1);
+      }
+    }
+    __syncwarp();   // the buffer is refilled by the next iteration's issue
 
-    int buf = 0;
-    for (int c = c_first; c < nch; c += kTcaWarps, buf ^= 1) {
-      if (c + kTcaWarps < nch) {
-        issue(c + kTcaWarps, buf ^ 1);
-        cp_async_wait<1>();
-      } else {
-        cp_async_wait<0>();
-      }
-      __syncwarp();
-      const int cnt = min(kTcaChunk, s1 - (s0 + c * kTcaChunk));
-      const bf16* Ks = wbuf + (size_t)buf * 2 * kTcaChunk * KROW;
-      const bf16* Vs = Ks + kTcaChunk * KROW;
-      // logits: 4 n-tiles of 8 positions
-      float s[4][2];
-#pragma unroll
-      for (int t = 0; t < 4; ++t) {
-        s[t][0] = s[t][1] = 0.f;
-        const bf16* kr = Ks + (size_t)(t * 8 + (lane & 7)) * KROW + 8 * (lane >> 3);
-#pragma unroll
-        for (int kk = 0; kk < KSTEPS; kk += 2) {
-          uint32_t b0, b1, b2, b3;
-          tca::ldsm_x4(kr + kk * 16, b0, b1, b2, b3);
-          tca::mma16816(s[t][0], s[t][1], z, qh[kk][0], qh[kk][1], b0, b1);
-          tca::mma16816(s[t][0], s[t][1], z, qh[kk + 1][0], qh[kk + 1][1], b2, b3);
-          if (SPLIT) {
-            tca::mma16816(s[t][0], s[t][1], z, ql[kk][0], ql[kk][1], b0, b1);
-            tca::mma16816(s[t][0], s[t][1], z, ql[kk + 1][0], ql[kk + 1][1], b2, b3);
-          }
-        }
-      }
-      // online softmax of row h0 over positions t*8 + c2 (+1)
-      float cm = -INFINITY;
-#pragma unroll
-      for (int t = 0; t < 4; ++t) {
-        if (t * 8 + c2 >= cnt) s[t][0] = -INFINITY;
-        if (t * 8 + c2 + 1 >= cnt) s[t][1] = -INFINITY;
-        cm = fmaxf(cm, fmaxf(s[t][0], s[t][1]));
-      }
-      cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, 1));
-      cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, 2));
-      const float mn = fmaxf(mrun, cm);
-      const float alpha = mrun == -INFINITY ? 0.f : expf(mrun - mn);
-      float ps = 0.f;
-#pragma unroll
-      for (int t = 0; t < 4; ++t) {
-        s[t][0] = expf(s[t][0] - mn);
-        s[t][1] = expf(s[t][1] - mn);
-        ps += s[t][0] + s[t][1];
-      }
-      ps += __shfl_xor_sync(0xffffffffu, ps, 1);
-      ps += __shfl_xor_sync(0xffffffffu, ps, 2);
-      lrun = lrun * alpha + ps;
-      mrun = mn;
-#pragma unroll
-      for (int t = 0; t < DT; ++t) {
-        o[t][0] *= alpha;
-        o[t][1] *= alpha;
-      }
-      // O += P V: two k-steps of 16 positions
-#pragma unroll
-      for (int k2 = 0; k2 < 2; ++k2) {
-        uint32_t ah0, ah2, al0 = 0, al2 = 0;
-        if (SPLIT) {
-          tca::split_pack(s[2 * k2][0], s[2 * k2][1], ah0, al0);
-          tca::split_pack(s[2 * k2 + 1][0], s[2 * k2 + 1][1], ah2, al2);
-        } else {
-          ah0 = tca::pack_bf16(s[2 * k2][0], s[2 * k2][1]);
-          ah2 = tca::pack_bf16(s[2 * k2 + 1][0], s[2 * k2 + 1][1]);
-        }
-        // lanes 0-7 / 8-15: positions 16*k2 + 0..7 / 8..15 of dims 8t..; 16-31: dims 8(t+1)..
-        const bf16* vr = Vs + (size_t)(k2 * 16 + (lane & 7) + 8 * ((lane >> 3) & 1)) * KROW + 8 * (lane >> 4);
-#pragma unroll
-        for (int t = 0; t < DT; t += 2) {
-          uint32_t b0, b1, b2, b3;
-          tca::ldsm_x4_t(vr + t * 8, b0, b1, b2, b3);
-          tca::mma16816(o[t][0], o[t][1], z, ah0, ah2, b0, b1);
-          tca::mma16816(o[t + 1][0], o[t + 1][1], z, ah0, ah2, b2, b3);
-          if (SPLIT) {
-            tca::mma16816(o[t][0], o[t][1], z, al0, al2, b0, b1);
-            tca::mma16816(o[t + 1][0], o[t + 1][1], z, al0, al2, b2, b3);
-          }
-        }
-      }
-      __syncwarp();   // the buffer is refilled by the issue two chunks on
-    }
-    // combine the four warps (the K/V buffers are free once all are done)
-    __syncthreads();
-    if ((lane & 3) == 0) {
-      mw[warp * 8 + h0] = mrun;
-      lw[warp * 8 + h0] = lrun;
-    }
-#pragma unroll
-    for (int t = 0; t < DT; ++t) {
-      float* d = ow + ((size_t)warp * 8 + h0) * HD + t * 8 + c2;
-      d[0] = o[t][0];
-      d[1] = o[t][1];
-    }
-    __syncthreads();
-    const size_t obase = (size_t)j * nq * HD + (size_t)g * G * HD;
-    for (int x = tid; x < G * HD; x += kTcaThreads) {
-      const int h = x / HD, e = x - h * HD;
-      float M = -INFINITY;
-#pragma unroll
-      for (int w = 0; w < kTcaWarps; ++w) M = fmaxf(M, mw[w * 8 + h]);
-      float L = 0.f, O = 0.f;
-#pragma unroll
-      for (int w = 0; w < kTcaWarps; ++w) {
-        const float mv = mw[w * 8 + h];
-        const float f = mv == -INFINITY ? 0.f : expf(mv - M);
-        L += lw[w * 8 + h] * f;
-        O += ow[((size_t)w * 8 + h) * HD + e] * f;
-      }
+    const TcaCursor cs = cc;   // the span this chunk belongs to
+    advance(cc, cnt);
+    xc += cnt;
+    if (cs.p + cnt == cs.np || xc == b) {
+      // end of the span: its stream covers flattened [S0, S0 + np), cut by the
+      // shares into spans first .. last (this warp's is gw - first)
+      const int S0 = pref[cs.j] + cs.g * cs.np;
+      const int first = S0 / share, nsp = (S0 + cs.np - 1) / share - first + 1;
+      const size_t obase = ((size_t)cs.j * nq + (size_t)cs.g * G) * HD;
+      // this lane: heads c2 + e (e = 0, 1), channels 16 t + h0 (+ 8)
       if (nsp == 1) {
-        store_out(A.out, A.out_lo, obase + x, O / L);
-      } else {
-        const size_t slot = ((size_t)j * nq + g * G + h) * A.max_spans + sp;
-        __stcg(A.part_acc + slot * HD + e, O);
-        if (e == 0) {
-          __stcg(A.part_m + slot, M);
-          __stcg(A.part_l + slot, L);
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          if (c2 + e < G) {
+            const float inv = 1.f / lrun[e];
+            const size_t ob = obase + (size_t)(c2 + e) * HD + h0;
+#pragma unroll
+            for (int t = 0; t < DT / 2; ++t) {
+              store_out(A.out, A.out_lo, ob + 16 * t, o[t][e] * inv);
+              store_out(A.out, A.out_lo, ob + 16 * t + 8, o[t][2 + e] * inv);
+            }
+          }
+        }
+      } else {   // a partial for attn_tc_merge_kernel
+        const int sp = gw - first;
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          if (c2 + e < G) {
+            const size_t slot = ((size_t)cs.j * nq + (size_t)cs.g * G + c2 + e) * A.max_spans + sp;
+            float* pa = A.part_acc + slot * HD + h0;
+#pragma unroll
+            for (int t = 0; t < DT / 2; ++t) {
+              __stcg(pa + 16 * t, o[t][e]);
+              __stcg(pa + 16 * t + 8, o[t][2 + e]);
+            }
+            if (h0 == 0) {
+              __stcg(A.part_m + slot, mrun[e]);
+              __stcg(A.part_l + slot, lrun[e]);
+            }
+          }
+        }
+        if (nsp <= kTcaWarpMerge) {
+          // the partial is visible before the arrival is counted; the warp
+          // that completes the stream merges (and re-arms the counter)
+          __syncwarp();
+          int last = 0;
+          if (lane == 0) {
+            __threadfence();
+            int32_t* ctr = A.ctr + cs.j * nkv + cs.g;
+            const int old = atomicAdd(ctr, 1);
+            last = old == nsp - 1;
+            if (last) *ctr = 0;
+            __threadfence();
+          }
+          last = __shfl_sync(0xffffffffu, last, 0);
+          __syncwarp();
+          if (last) attn_tc_warp_merge<HD>(A, cs.j, cs.g, nsp, obase, lane);
         }
       }
     }
-    if (nsp > 1) {
-      __syncthreads();
-      if (tid == 0) {
-        __threadfence();
-        const int old = atomicAdd(&A.ctr[j * nkv + g], 1);
-        *last_s_p = (old == nsp - 1);
-        if (*last_s_p) A.ctr[j * nkv + g] = 0;
-        __threadfence();
-      }
-      __syncthreads();
-      if (*last_s_p) attn_span_merge<bf16, HD, kTcaThreads>(A, j, g, nsp, obase, tid);
-    }
-    __syncthreads();
   }
-  if (!waited) {
-    pdl_wait();
-    pdl_trigger();
-  }
+}
+
+// Merge of the span partials of stream (row j, KV head g) = (blockIdx.x /
+// nkv, blockIdx.x % nkv), in span order, for streams the attention kernel cut
+// into more than kTcaWarpMerge spans.
+template <int HD>
+__device__ __forceinline__ void attn_tc_merge_run(const AttnArgs<bf16>& A) {
+  const int m = A.count ? *A.count : A.n;
+  const int j = blockIdx.x / A.nkv, g = blockIdx.x - j * A.nkv;
+  if (j >= m || *reinterpret_cast<const volatile int32_t*>(A.status + 1) != 0) return;
+  const int np = (A.meta[j + 1] - A.meta[j]) / A.nkv, share = A.meta[m + 1];
+  const int S0 = A.meta[j] + g * np;
+  const int nsp = (S0 + np - 1) / share - S0 / share + 1;
+  if (nsp <= kTcaWarpMerge) return;   // written out, or merged in the attention kernel
+  const size_t obase = ((size_t)j * A.nq + (size_t)g * (A.nq / A.nkv)) * HD;
+  attn_span_merge<bf16, HD, kTcaMergeThreads, true>(A, j, g, nsp, obase, threadIdx.x);
 }
 
 }  // namespace buddy

@@ -100,7 +100,9 @@ void launch_qkv_finalize(const Ctx& c, const float* qkv, const float* bias, RowS
                          cudaStream_t s);
 void launch_attention(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q,
                       void* attn_out, void* attn_lo, cudaStream_t s);   // attention.cu
-int attention_chunk();
+int attention_max_spans(int max_pos);   // span partials per (row, query head)
+bool attention_tc(const Ctx& c);         // tensor-core loop: launch_attention_merge follows
+void launch_attention_merge(const Ctx& c, RowSel sel, void* out, void* out_lo, cudaStream_t s);
 void launch_route(const Ctx& c, int B, const float* h1, const float* pool, const int32_t* len,
                   int len_bias, const int32_t* k, uint8_t* mask, int32_t* sel, float* scores,
                   cudaStream_t s);
@@ -148,11 +150,12 @@ struct Ctx {
   void* attn_lo = nullptr;     // [maxB, qd]
   float* qkv = nullptr;        // [maxB, qkvN]
   float* q = nullptr;          // [maxB, qd]
-  int attn_chunk = 128, attn_max_chunks = 1;
+  int attn_max_chunks = 1;   // span partial slots per (row, query head)
   float* attn_m = nullptr;     // [maxB, nq, max_chunks]
   float* attn_l = nullptr;
   float* attn_acc = nullptr;   // [maxB, nq, max_chunks, hd]
   int32_t* attn_ctr = nullptr; // [maxB, nkv] chunk arrivals (self-resetting)
+  int32_t* attn_meta = nullptr;   // [maxB + 2] row prefix and share (tensor-core attention)
   float* dm_u = nullptr;       // [maxB, r]
   uint8_t* mask = nullptr;     // [maxB, L]
   int32_t* sel = nullptr;      // [maxB, Lm]
