@@ -360,14 +360,24 @@ __device__ __forceinline__ void tc_apply4(const TcParams& p, int tile, int j, in
   }
 }
 
+// Position (in float4 units) of row j's 4-column group at column c in a
+// workspace slot.  Up to 16 rows a slot is row-major (the groups of a row
+// contiguous: the few rows' items are read group by group); above, group-major
+// (a group's rows contiguous: the 32 lanes of a warp hold 32 rows of an
+// accumulator column block, and store 512 contiguous bytes per group).
+__device__ __forceinline__ size_t tc_ws_idx(const TcParams& p, int j, int c) {
+  return p.rows_max <= 16 ? (size_t)j * (p.bw >> 2) + (c >> 2) : (size_t)(c >> 2) * p.rows_max + j;
+}
+
 // One epilogue item (row j, 4-column group at c of `tile`): the partials of
 // all K splits (and of the partner columns) are summed in split order, eight
 // splits' loads in flight at a time, and the epilogue is applied.
 template <int EPI, bool SPLIT>
 __device__ __forceinline__ void tc_fix_item(const TcParams& p, int tile, int j, int c) {
   const int po = tc_partner_off<EPI>(p);
-  const size_t sstride = (size_t)p.n_tiles * p.rows_max * p.bw;   // one split's slots
-  const float* sl = p.ws + ((size_t)tile * p.rows_max + j) * p.bw + c;
+  const size_t sstride = (size_t)p.n_tiles * p.rows_max * p.bw / 4;   // one split's slots (float4)
+  const size_t pstride = tc_ws_idx(p, j, c + po) - tc_ws_idx(p, j, c);
+  const float4* sl = reinterpret_cast<const float4*>(p.ws + (size_t)tile * p.rows_max * p.bw) + tc_ws_idx(p, j, c);
   float v[4] = {0.f, 0.f, 0.f, 0.f}, vp[4] = {0.f, 0.f, 0.f, 0.f}, rs[4] = {0.f, 0.f, 0.f, 0.f};
   if (EPI == EPI_RESID) {
     const int seq = p.rows ? p.rows[j] : j;
@@ -381,8 +391,8 @@ __device__ __forceinline__ void tc_fix_item(const TcParams& p, int tile, int j, 
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
       if (s0 + k < p.splits) {
-        x[k] = __ldcg(reinterpret_cast<const float4*>(sl + (size_t)(s0 + k) * sstride));
-        if (po) y[k] = __ldcg(reinterpret_cast<const float4*>(sl + (size_t)(s0 + k) * sstride + po));
+        x[k] = __ldcg(sl + (size_t)(s0 + k) * sstride);
+        if (po) y[k] = __ldcg(sl + (size_t)(s0 + k) * sstride + pstride);
       }
     }
 #pragma unroll
@@ -413,7 +423,7 @@ __device__ __forceinline__ void tc_epilogue_unit(const TcParams& p, int u, int m
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int q = warp & 3;   // TMEM lane quarter this warp may access
   const int tile = u % p.n_tiles;
-  float* slot = p.ws + (size_t)u * p.rows_max * p.bw;
+  float4* slot = reinterpret_cast<float4*>(p.ws + (size_t)u * p.rows_max * p.bw);
   for (int t = 0; t < p.mt; ++t) {
     if (t * 128 + q * 32 >= m) continue;   // warp-uniform
     const int j = t * 128 + q * 32 + lane;
@@ -422,9 +432,9 @@ __device__ __forceinline__ void tc_epilogue_unit(const TcParams& p, int u, int m
       float v[64];
       ptx::tmem_ld64(ta + c0, v);
       if (j < m) {
-        float4* d = reinterpret_cast<float4*>(slot + (size_t)j * p.bw + c0);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) __stcg(d + i, make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]));
+        for (int i = 0; i < 16; ++i)
+          __stcg(slot + tc_ws_idx(p, j, c0 + 4 * i), make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]));
       }
     }
   }

@@ -274,8 +274,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // Deferred fixup of a GEMM whose units only staged their partials: items
 // (tile, row, 4-column group) over the whole grid, each summing its splits in
 // split order (the same order, hence the same result, as the in-kernel
-// finisher) and applying the epilogue.  Consecutive threads take consecutive
-// column groups of a row, so the workspace reads are coalesced.
+// finisher) and applying the epilogue.  With row-major slots consecutive
+// threads take consecutive groups of a row; with group-major slots a warp
+// takes 8 rows x 4 groups (128 contiguous bytes of each group's partials,
+// 4 contiguous groups of each row's outputs).
 template <int EPI, bool SPLIT>
 __global__ void __launch_bounds__(kTcFixThreads) gemm_fix_kernel(const TcParams p) {
   pdl_wait();
@@ -284,13 +286,27 @@ __global__ void __launch_bounds__(kTcFixThreads) gemm_fix_kernel(const TcParams 
   const int m = p.count ? *p.count : p.n;
   if (m <= 0) return;
   const int ng = tc_groups<EPI>(p);
-  const long long items = (long long)p.n_tiles * m * ng;
-  for (long long it = (long long)blockIdx.x * kTcFixThreads + threadIdx.x; it < items;
-       it += (long long)gridDim.x * kTcFixThreads) {
-    const int g = (int)(it % ng);
-    const long long r = it / ng;
-    const int j = (int)(r % m), tile = (int)(r / m);
-    tc_fix_item<EPI, SPLIT>(p, tile, j, tc_group_col<EPI>(p, g));
+  const long long stride = (long long)gridDim.x * kTcFixThreads;
+  if (p.rows_max <= 16) {
+    const long long items = (long long)p.n_tiles * m * ng;
+    for (long long it = (long long)blockIdx.x * kTcFixThreads + threadIdx.x; it < items; it += stride) {
+      const int g = (int)(it % ng);
+      const long long r = it / ng;
+      const int j = (int)(r % m), tile = (int)(r / m);
+      tc_fix_item<EPI, SPLIT>(p, tile, j, tc_group_col<EPI>(p, g));
+    }
+  } else {
+    // warp blocks of 8 rows x 4 groups (ng is a multiple of 4)
+    const int rb = (m + 7) >> 3, gb = ng >> 2;
+    const long long items = (long long)p.n_tiles * gb * rb * 32;
+    const int lane = threadIdx.x & 31;
+    for (long long it = (long long)blockIdx.x * kTcFixThreads + threadIdx.x; it < items; it += stride) {
+      const long long wb = it >> 5;
+      const int j = (int)(wb % rb) * 8 + (lane & 7);
+      const long long r = wb / rb;
+      const int g = (int)(r % gb) * 4 + (lane >> 3), tile = (int)(r / gb);
+      if (j < m) tc_fix_item<EPI, SPLIT>(p, tile, j, tc_group_col<EPI>(p, g));
+    }
   }
 }
 
