@@ -3,17 +3,22 @@
 // attend over positions 0..len[i] of that head's cache (the new token included;
 // zero-filled positions of earlier skipped steps take part with logit 0).
 //
-// Work items are (row, KV head, span of P positions); P is derived on the
-// device from the total number of positions so that there are about as many
-// items as half the grid (64 <= P <= 1024).  Persistent CTAs walk the items.
-// Inside an item the CTA streams chunks of 64 positions: K and V are copied
-// into shared memory with 16-byte cp.async (double-buffered: the next chunk is
-// in flight while the current one is used; K rows padded so that lanes reading
-// 32 different positions hit distinct banks), then logits, an online softmax
-// and P.V run in fp32.  An item covering the whole row writes the output;
-// otherwise it writes a partial (running max, sum of exponentials,
-// unnormalised output) and the last item of the (row, head) to finish merges
-// the partials in span order (log-sum-exp) and writes the output.
+// Two work loops:
+//   * bf16 caches (G <= 8): the tensor-core loop of attn_tc.cuh (warp shares
+//     of the concatenated position streams, mma.sync contractions) and its
+//     span-merge kernel;
+//   * fp32 caches (and the opt-in per-layer persistent kernel): the CUDA-core
+//     loop of attn_common.cuh.  Its work items are (row, KV head, span of P
+//     positions); P is derived on the device from the total number of
+//     positions so that there are about as many items as half the grid
+//     (64 <= P <= 1024).  Persistent CTAs walk the items.  Inside an item the
+//     CTA streams chunks of 64 positions: K and V are copied into shared
+//     memory with 16-byte cp.async (double-buffered; K rows padded so that
+//     lanes reading 32 different positions hit distinct banks), then logits,
+//     an online softmax and P.V run in fp32.  An item covering the whole row
+//     writes the output; otherwise it writes a partial (running max, sum of
+//     exponentials, unnormalised output) and the last item of the (row, head)
+//     to finish merges the partials in span order (log-sum-exp).
 #include <cuda_runtime.h>
 
 #include <algorithm>

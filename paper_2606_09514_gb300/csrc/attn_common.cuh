@@ -1,5 +1,6 @@
-// Decode attention work loop shared by the attention kernel and the
-// per-layer persistent kernel (see attention.cu for the algorithm).
+// CUDA-core decode attention work loop, shared by the fp32 attention kernel
+// and the per-layer persistent kernel (see attention.cu for the algorithm),
+// and the span merge used by both attention loops.
 #pragma once
 
 #include <cuda_runtime.h>
