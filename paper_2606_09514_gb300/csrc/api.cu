@@ -55,7 +55,7 @@ static void free_ctx(buddy_ctx* x) {
   void* ptrs[] = {c.rope_cos, c.rope_sin, c.status, c.xn, c.act, c.attn_out, c.qkv, c.q,
                   c.attn_m, c.attn_l, c.attn_acc, c.attn_ctr, c.dm_u, c.mask, c.sel, c.scores, c.rows,
                   c.count, c.h_in_stage, c.h_out_stage, c.k_stage, c.mask_stage, c.xn_lo, c.act_lo, c.attn_lo, c.lk_bar,
-                  c.gemm_ws, c.gemm_ctr};
+                  c.gemm_ws, c.gemm_ctr, c.attn_meta};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   if (x->cap_stream) cudaStreamDestroy(x->cap_stream);
