@@ -20,11 +20,19 @@
 // bytes that follow within the stage (their results are discarded).
 //
 // The accumulator of a unit (tile, K split) is mt x 256 fp32 TMEM columns.
-// Small batches use a short ring (about 100 KiB) and one accumulator, so that
-// two GEMM CTAs fit on an SM: under programmatic dependent launch the next
-// GEMM's CTAs start streaming their weights while the current one finishes.
-// Otherwise the ring fills shared memory and, with one M-tile, two
-// accumulators let the MMAs of the next unit overlap the epilogue.
+// The ring fills shared memory and, with one M-tile, two accumulators let the
+// MMAs of the next unit overlap the epilogue.  (BUDDY_TC_DUAL=1 instead gives
+// small batches a short ring and one accumulator so that two GEMM CTAs fit on
+// an SM; measured slower, kept opt-in.)
+//
+// Panel mode (up to 8 rows): the ring holds weight tiles only and the
+// activations of the QKV and gate/up GEMMs are the RMSNorm of the fp32
+// residual rows, computed by the epilogue warps into a shared-memory panel.
+//
+// Split-K: every unit stages its accumulator rows in a workspace slot; up to
+// 8 rows the last split of a tile to arrive sums the slots in split order
+// and applies the epilogue, above 8 rows gemm_fix_kernel does so over all
+// SMs (tc_ws_idx gives the slot layout).
 #pragma once
 
 #include <cuda.h>
