@@ -41,6 +41,7 @@
 
 #include "attn_common.cuh"
 #include "common.cuh"
+#include "ptx.cuh"
 
 namespace buddy {
 
@@ -532,12 +533,10 @@ __device__ __forceinline__ void attn_tc_run(const AttnArgs<bf16>& A, int cta, in
           __syncwarp();
           int last = 0;
           if (lane == 0) {
-            __threadfence();
             int32_t* ctr = A.ctr + cs.j * nkv + cs.g;
-            const int old = atomicAdd(ctr, 1);
+            const int old = ptx::atom_add_acq_rel(ctr, 1);
             last = old == nsp - 1;
-            if (last) *ctr = 0;
-            __threadfence();
+            if (last) *ctr = 0;   // re-armed for a later launch
           }
           last = __shfl_sync(0xffffffffu, last, 0);
           __syncwarp();

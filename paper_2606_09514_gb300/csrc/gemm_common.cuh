@@ -452,19 +452,18 @@ __device__ __forceinline__ void tc_epilogue_unit(const TcParams& p, int u, int m
   epi_bar();
   const int et = threadIdx.x & 127;
   if (et == 0) {
-    __threadfence();
+    // release of this CTA's slot (stored before the barrier) and, for the
+    // last arriver, acquire of the other splits' slots
     int last = 1;
     if (p.splits > 1) {
-      const int old = atomicAdd(&p.ctr[tile], 1);
+      const int old = ptx::atom_add_acq_rel(&p.ctr[tile], 1);
       last = old == p.splits - 1;
-      if (last) p.ctr[tile] = 0;
+      if (last) p.ctr[tile] = 0;   // re-armed for a later launch
     }
     *last_flag = last;
-    __threadfence();
   }
   epi_bar();
   if (*last_flag) {
-    __threadfence();
     const int ng = tc_groups<EPI>(p);
     const int items = m * ng;
     for (int it = et; it < items; it += 128) {   // one item per thread per round

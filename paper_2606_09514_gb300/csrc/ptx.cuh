@@ -8,6 +8,15 @@
 namespace buddy {
 namespace ptx {
 
+// Atomic add at GPU scope with acquire-release semantics: the caller's earlier
+// writes (and those ordered before it by a barrier) are visible to whoever
+// observes the new value, and later reads see what the observed writers wrote.
+__device__ __forceinline__ int atom_add_acq_rel(int* p, int v) {
+  int old;
+  asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
