@@ -33,7 +33,7 @@ METRIC = "budget-routed decode tokens/s at 1 GB300 per budget; % of HBM/tensor r
 # ncu dram bytes (read + write) per launch of the dominant kernel, from the
 # committed ncu summary of the gate/up GEMM (3-layer model with the same layer
 # shapes as the 32-layer bench workload); absent for kernels not captured
-NCU_TRAFFIC_PER_LAUNCH = {"gemm_gate_up": 238094336}
+NCU_TRAFFIC_PER_LAUNCH = {"gemm_gate_up": 238353664}
 
 
 def _peaks():
