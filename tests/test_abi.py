@@ -91,3 +91,18 @@ def test_ctypes_structs_match_c_layout():
         assert int(got[n]) == ctypes.sizeof(cls), n
         for f, _ in cls._fields_:
             assert int(got[f"{n}.{f}"]) == getattr(cls, f).offset, (n, f)
+
+
+def test_profiler_class_names_match_binding(lib):
+    """The binding's names for the profiler's kernel classes are the library's,
+    in the order of the header's enum."""
+    from paper_2606_09514_gb300 import binding
+    txt = open(HEADER).read()
+    enum = re.search(r"enum\s*\{\s*(BUDDY_PROF_CHECK[^}]*)\}", txt).group(1)
+    n_cls = len(re.findall(r"\bBUDDY_PROF_(?!NCLASS)\w+", enum))
+    assert n_cls == len(binding.PROF_CLASSES)
+    lib.buddy_profile_class_name.restype = ctypes.c_char_p
+    lib.buddy_profile_class_name.argtypes = [ctypes.c_int32]
+    names = [lib.buddy_profile_class_name(i).decode() for i in range(n_cls)]
+    assert names == binding.PROF_CLASSES
+    assert lib.buddy_profile_class_name(n_cls).decode() == "unknown"
