@@ -32,7 +32,8 @@ def to_f64(t: torch.Tensor) -> np.ndarray:
 
 def oracle_shape(s: ModelShape) -> O.Shape:
     return O.Shape(s.n_layers, s.d_model, s.n_q_heads, s.n_kv_heads, s.head_dim, s.ffn_dim,
-                   s.dm_hidden, s.dtype, s.rms_eps, s.rope_theta)
+                   s.dm_hidden, s.dtype, s.rms_eps, s.rope_theta, feature=s.feature,
+                   ctx_layer=s.ctx_layer, skip_kv=s.skip_kv)
 
 
 def layer_from_tensors(w: Dict[str, torch.Tensor]) -> O.LayerWeights:
@@ -45,7 +46,7 @@ def layer_from_tensors(w: Dict[str, torch.Tensor]) -> O.LayerWeights:
 
 def build_model(shape: ModelShape, seed: int, *, layer_source=None, dm_source=None,
                 prior: Optional[torch.Tensor] = None, omega: float = 0.0,
-                cache_layers: int = 4) -> O.Model:
+                cache_layers: int = 4, predictor_source=None) -> O.Model:
     """Oracle model for a generated workload.  `layer_source(l)` may supply the
     generator's tensors (e.g. already generated on the GPU and copied back);
     by default they are generated on the host."""
@@ -59,7 +60,12 @@ def build_model(shape: ModelShape, seed: int, *, layer_source=None, dm_source=No
     dm = O.DecisionModule(w1=to_f64(dmw["w1"]), b1=to_f64(dmw["b1"]), w2=to_f64(dmw["w2"]),
                           b2=to_f64(dmw["b2"]),
                           prior=None if prior is None else to_f64(prior), omega=float(omega))
-    return O.Model(oracle_shape(shape), layer, dm)
+    bp = None
+    if shape.predictor_hidden > 0:
+        pw = predictor_source() if predictor_source is not None else synth.predictor_weights(shape, seed, "cpu")
+        bp = O.BudgetPredictor(w1=to_f64(pw["w1"]), b1=to_f64(pw["b1"]), w2=to_f64(pw["w2"]),
+                               b2=to_f64(pw["b2"]))
+    return O.Model(oracle_shape(shape), layer, dm, bp)
 
 
 def build_state(shape: ModelShape, seed: int, n_ctx: Sequence[int],

@@ -23,8 +23,10 @@ KV_TOL = HIDDEN_TOL
 
 
 def adopt_routes(o_scores: np.ndarray, o_sel: Sequence[Sequence[int]], g_sel: Sequence[Sequence[int]],
-                 k: Sequence[int]) -> Tuple[List[List[int]], List[str], int]:
-    """Returns (sets the oracle continues with, failures, number adopted)."""
+                 k: Sequence[int], first: int = 1) -> Tuple[List[List[int]], List[str], int]:
+    """Returns (sets the oracle continues with, failures, number adopted).
+    o_scores[i][j] belongs to layer first + j; k[i] is the budget the
+    sequence used (the set sizes decide it where k[i] is 0, i.e. predicted)."""
     out, fails, adopted = [], [], 0
     for i, (os_, gs) in enumerate(zip(o_sel, g_sel)):
         os_, gs = sorted(int(x) for x in os_), sorted(int(x) for x in gs)
@@ -32,7 +34,7 @@ def adopt_routes(o_scores: np.ndarray, o_sel: Sequence[Sequence[int]], g_sel: Se
             out.append(os_)
             continue
         s = np.asarray(o_scores[i], dtype=np.float64)
-        ki = int(k[i])
+        ki = int(k[i]) if int(k[i]) > 0 else len(os_)
         srt = np.sort(s)[::-1]
         if len(gs) != ki or ki >= len(s):
             fails.append(f"seq {i}: gpu {gs} vs oracle {os_} (k={ki})")
@@ -41,7 +43,7 @@ def adopt_routes(o_scores: np.ndarray, o_sel: Sequence[Sequence[int]], g_sel: Se
         kth = srt[ki - 1]
         gap = srt[ki - 1] - srt[ki]
         diff = set(os_) ^ set(gs)
-        near = all(abs(s[l - 1] - kth) < ROUTE_MARGIN for l in diff)
+        near = all(abs(s[l - first] - kth) < ROUTE_MARGIN for l in diff)
         if gap < ROUTE_MARGIN and near:
             out.append(gs)
             adopted += 1
@@ -57,6 +59,6 @@ def max_rel_err(g: np.ndarray, o: np.ndarray) -> float:
     return float(np.max(np.abs(g - o)) / max(np.max(np.abs(o)), 1e-30))
 
 
-def sel_from_mask(mask: np.ndarray) -> List[List[int]]:
+def sel_from_mask(mask: np.ndarray, first: int = 1) -> List[List[int]]:
     L = mask.shape[1]
-    return [[l for l in range(1, L - 1) if mask[i, l]] for i in range(mask.shape[0])]
+    return [[l for l in range(first, L - 1) if mask[i, l]] for i in range(mask.shape[0])]

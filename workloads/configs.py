@@ -32,10 +32,24 @@ class ModelShape:
     rope_theta: float
     qkv_bias: bool = False
     random_norm: bool = False   # test shapes draw RMSNorm gains instead of using 1
+    # router variants (Sec. 4.3, Sec. 5.4 ablations, Sec. 6)
+    feature: str = "v"          # planner feature: "v", "k" or "kv" (K + V)
+    ctx_layer: int = 0          # c: layers 0..c always run, the planner reads layer c
+    skip_kv: str = "zero"       # "zero" (zero-filled K/V at skipped layers) or "masked"
+    predictor_hidden: int = 0   # Budget Predictor hidden width (0: no predictor)
 
     @property
     def l_mid(self) -> int:
         return self.n_layers - 2
+
+    @property
+    def n_cand(self) -> int:
+        """Routed candidate layers c+1 .. L-2."""
+        return self.n_layers - 2 - self.ctx_layer
+
+    @property
+    def first_candidate(self) -> int:
+        return self.ctx_layer + 1
 
     @property
     def kv_dim(self) -> int:
@@ -84,7 +98,8 @@ class Workload:
         return _draw_meta(self)[0]
 
     def budgets(self) -> np.ndarray:
-        """Per-sequence budget k_i in [1, L_mid] (int64, seeded)."""
+        """Per-sequence budget k_i in [1, n_cand], or 0 where the Budget
+        Predictor chooses it (int64, seeded)."""
         return _draw_meta(self)[1]
 
     def capacities(self, extra_steps: int = 0) -> np.ndarray:
@@ -110,7 +125,7 @@ def _draw_meta(w: Workload):
         assert ctx.shape == (B,)
     else:
         raise ValueError(w.ctx_kind)
-    Lm = w.shape.l_mid
+    Lm = w.shape.n_cand
     if w.k_kind == "fixed":
         k = np.full(B, int(w.k_args[0]), dtype=np.int64)
     elif w.k_kind == "choice":
@@ -123,7 +138,10 @@ def _draw_meta(w: Workload):
         assert k.shape == (B,)
     else:
         raise ValueError(w.k_kind)
-    assert np.all((k >= 1) & (k <= Lm)), "budgets must lie in [1, L_mid]"
+    ok = (k >= 1) & (k <= Lm)
+    if w.shape.predictor_hidden > 0:
+        ok |= k == 0
+    assert np.all(ok), "budgets must lie in [1, n_cand] (0: predicted)"
     return ctx, k
 
 
@@ -194,7 +212,39 @@ P_QWEN_3L_B256 = Workload("qwen2.5-7b-3layer-b256",
                           batch=256, steps=8, seed=0, ctx_kind="lognormal", ctx_args=(2048, 0.5, 512, 8192),
                           k_kind="fixed", k_args=(1,))
 
-BY_NAME = {w.name: w for w in FULL_WORKLOADS + [T_GQA, T_QWEN, T_F32, P_LLAMA3_3L_B1, P_QWEN_3L_B256]}
+# Router variants on the small shapes: K and K + V planner features, a context
+# layer c > 0, the masked skip-KV variant, and the Budget Predictor (budget 0 =
+# predicted).
+T_PRED = Workload("t-small-f32-pred", dataclasses.replace(SMALL_F32, name="small-f32-pred", predictor_hidden=24),
+                  batch=6, steps=2, seed=3, ctx_kind="list", ctx_args=(0, 7, 64, 129, 31, 300),
+                  k_kind="list", k_args=(0, 2, 0, 3, 0, 0))
+T_VARIANTS = [
+    Workload("t-gqa-bf16-k", dataclasses.replace(SMALL_GQA_BF16, name="small-gqa-bf16-k", feature="k"),
+             batch=37, steps=3, seed=1, ctx_kind="uniform", ctx_args=(0, 300), k_kind="uniform", k_args=(1, 4)),
+    Workload("t-qwen-bf16-kv-c1-pred",
+             dataclasses.replace(SMALL_QWEN_BF16, name="small-qwen-bf16-kv-c1-pred", feature="kv", ctx_layer=1,
+                                 predictor_hidden=40),
+             batch=19, steps=3, seed=2, ctx_kind="list",
+             ctx_args=(0, 1, 2, 63, 64, 65, 127, 128, 129, 255, 256, 257, 511, 700, 5, 17, 1000, 333, 90),
+             k_kind="list", k_args=(1, 0, 3, 2, 4, 0, 1, 0, 2, 3, 4, 0, 4, 2, 3, 1, 0, 2, 3)),
+    Workload("t-gqa-bf16-masked", dataclasses.replace(SMALL_GQA_BF16, name="small-gqa-bf16-masked", skip_kv="masked"),
+             batch=37, steps=3, seed=1, ctx_kind="uniform", ctx_args=(0, 300), k_kind="uniform", k_args=(1, 4)),
+    Workload("t-small-f32-masked-c2-kv",
+             dataclasses.replace(SMALL_F32, name="small-f32-masked-c2-kv", skip_kv="masked", ctx_layer=2,
+                                 feature="kv", n_layers=7),
+             batch=6, steps=2, seed=3, ctx_kind="list", ctx_args=(0, 7, 64, 129, 31, 300),
+             k_kind="list", k_args=(1, 2, 3, 3, 2, 1)),
+]
+
+BY_NAME = {w.name: w for w in FULL_WORKLOADS + [T_GQA, T_QWEN, T_F32, T_PRED, P_LLAMA3_3L_B1, P_QWEN_3L_B256]
+           + T_VARIANTS}
+
+
+def with_shape(w: Workload, name: Optional[str] = None, **shape_changes) -> Workload:
+    """The same workload on a shape with some fields changed (router variants)."""
+    sh = dataclasses.replace(w.shape, name=w.shape.name + "-" + "-".join(f"{k}{v}" for k, v in shape_changes.items()),
+                             **shape_changes)
+    return dataclasses.replace(w, shape=sh, name=name or f"{w.name}-{sh.name}")
 
 
 def scaled(w: Workload, *, batch: Optional[int] = None, steps: Optional[int] = None,

@@ -34,6 +34,7 @@ _CHUNK_GPU = 1 << 25
 KIND = {"w_q": 1, "w_k": 2, "w_v": 3, "w_o": 4, "w_gate": 5, "w_up": 6, "w_down": 7,
         "b_q": 8, "b_k": 9, "b_v": 10, "attn_norm": 11, "ffn_norm": 12,
         "dm_w1": 20, "dm_b1": 21, "dm_w2": 22, "dm_b2": 23, "prior": 24,
+        "bp_w1": 25, "bp_b1": 26, "bp_w2": 27, "bp_b2": 28,
         "k_cache": 30, "v_cache": 31, "h_in": 40}
 
 WEIGHT_STD = 0.02
@@ -142,16 +143,26 @@ def layer_weights(shape: ModelShape, seed: int, layer: int, device="cpu") -> Dic
 
 
 def dm_weights(shape: ModelShape, seed: int, device="cpu") -> Dict[str, torch.Tensor]:
-    """Decision Module (Linear 2d->r, SiLU, Linear r->L_mid), fp32."""
-    d, r, Lm = shape.d_model, shape.dm_hidden, shape.l_mid
+    """Decision Module (Linear 2d->r, SiLU, Linear r->n_cand), fp32."""
+    d, r, Lm = shape.d_model, shape.dm_hidden, shape.n_cand
     g = lambda kind, shp: normal(shp, stream_key(seed, kind), WEIGHT_STD, torch.float32, device)
     return {"w1": g("dm_w1", (r, 2 * d)), "b1": g("dm_b1", (r,)),
             "w2": g("dm_w2", (Lm, r)), "b2": g("dm_b2", (Lm,))}
 
 
+def predictor_weights(shape: ModelShape, seed: int, device="cpu") -> Dict[str, torch.Tensor]:
+    """Budget Predictor (Linear 2d->r_p, SiLU, Linear r_p->n_cand), fp32.  Its
+    second layer is drawn wider (sigma 0.5) so that the argmax varies across
+    inputs instead of being fixed by the bias."""
+    d, r, Lm = shape.d_model, shape.predictor_hidden, shape.n_cand
+    g = lambda kind, shp, sd=WEIGHT_STD: normal(shp, stream_key(seed, kind), sd, torch.float32, device)
+    return {"w1": g("bp_w1", (r, 2 * d)), "b1": g("bp_b1", (r,)),
+            "w2": g("bp_w2", (Lm, r), 0.5), "b2": g("bp_b2", (Lm,))}
+
+
 def prior(shape: ModelShape, seed: int, device="cpu") -> torch.Tensor:
-    """An arbitrary normalised prior vector p~ over the middle layers (fp32)."""
-    return normal((shape.l_mid,), stream_key(seed, "prior"), 1.0, torch.float32, device)
+    """An arbitrary normalised prior vector p~ over the routed layers (fp32)."""
+    return normal((shape.n_cand,), stream_key(seed, "prior"), 1.0, torch.float32, device)
 
 
 def kv_block(shape: ModelShape, seed: int, which: str, layer: int, seq: int,
