@@ -164,18 +164,20 @@ def oracle_sample(w, n_layers_sample=None, steps=1, device="cuda"):
     for t in range(steps):
         h = A.to_f64(synth.h_in(s, w.seed, t, [seq], device))
         prep0 = prep["t"]
+        info = {}
+
+        def truncate(rr):
+            info["full"] = len(rr.sel[0])
+            keep = rr.sel[0][:n_layers_sample]
+            info["keep"] = len(keep)
+            return [keep]
+
         t0 = time.perf_counter()
-        route = O.first_layer_and_route(model, st, h, k)
-        if n_layers_sample is not None:
-            keep = route.sel[0][:n_layers_sample]
-            full = len(route.sel[0])
-            route.sel = [keep]
-        res = O.routed_layers(model, st, route)
-        O.advance(st, res)
+        O.decode_step(model, st, h, k, override_sel=truncate if n_layers_sample is not None else None)
         dt = time.perf_counter() - t0 - (prep["t"] - prep0)
         total += dt
         if n_layers_sample is not None:
-            scaled_total += dt * (full + 2) / (len(keep) + 2)
+            scaled_total += dt * (info["full"] + 2) / (info["keep"] + 2)
         else:
             scaled_total += dt
     return {"seconds": total, "scaled_seconds": scaled_total, "tokens": steps,
@@ -329,8 +331,8 @@ def run_ours(args, ws, rank, local):
     # the timed steps launch every middle layer (a layer no row selected exits
     # at once); the profiled steps launch only the selected ones
     per_layer = ("rmsnorm", "gemm_qkv", "qkv_finalize", "attention", "gemm_o", "gemm_gate_up", "gemm_down",
-                 "layer", "gemm_fixup", "attn_merge")
-    exec_layers = (prof.get("attention", (0, 0))[1] + prof.get("layer", (0, 0))[1]) / prof_steps
+                 "gemm_fixup", "attn_merge")
+    exec_layers = prof.get("attention", (0, 0))[1] / prof_steps
     per_layer_kernels = sum(prof.get(k, (0, 0))[1] for k in per_layer) / max(exec_layers * prof_steps, 1)
     graph_extra = max(s.n_layers - exec_layers, 0) * per_layer_kernels
     out = {

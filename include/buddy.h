@@ -180,8 +180,11 @@ BUDDY_API int buddy_route(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t batc
  * process exits.  batch * dm_hidden must not exceed 65536, else
  * BUDDY_ERR_RANGE.  The first call on each device looks up the array's
  * device address (cudaGetSymbolAddress); make that first call outside any
- * stream capture.  All calls share the array: calls whose kernels overlap on
- * the GPU (different streams without ordering) race.  Allocates nothing. */
+ * stream capture.  The address is cached for the life of the process: after
+ * cudaDeviceReset (or anything else that recreates the device's primary
+ * context) the library must be reloaded before this entry is called again.
+ * All calls share the array: calls whose kernels overlap on the GPU
+ * (different streams without ordering) race.  Allocates nothing. */
 BUDDY_API int buddy_route_noalloc(int32_t n_layers, int32_t d_model, int32_t n_q_heads,
                                   int32_t n_kv_heads, int32_t head_dim, int32_t dm_hidden,
                                   const buddy_dm_weights* dm, int32_t batch, const float* pool_sum,
@@ -224,7 +227,6 @@ enum {
   BUDDY_PROF_CHECK = 0, BUDDY_PROF_RMSNORM, BUDDY_PROF_GEMM_QKV, BUDDY_PROF_QKV_FINALIZE,
   BUDDY_PROF_ATTENTION, BUDDY_PROF_GEMM_O, BUDDY_PROF_GEMM_GATE_UP, BUDDY_PROF_GEMM_DOWN,
   BUDDY_PROF_ROUTE, BUDDY_PROF_COMPACT, BUDDY_PROF_OTHER,
-  BUDDY_PROF_LAYER,   /* a whole block as one persistent kernel (small batches) */
   BUDDY_PROF_GEMM_FIXUP,   /* split-K sums + epilogues of the GEMMs (larger batches) */
   BUDDY_PROF_ATTN_MERGE,   /* span merge of the tensor-core attention */
   BUDDY_PROF_NCLASS

@@ -22,7 +22,7 @@ EXPORTED = ["buddy_create", "buddy_destroy", "buddy_set_weights", "buddy_kv_appe
             "buddy_set_profiling", "buddy_profile_read", "buddy_profile_class_name",
             "buddy_route_noalloc"]
 PROF_CLASSES = ["check", "rmsnorm", "gemm_qkv", "qkv_finalize", "attention", "gemm_o", "gemm_gate_up",
-                "gemm_down", "route", "compact", "other", "layer", "gemm_fixup",
+                "gemm_down", "route", "compact", "other", "gemm_fixup",
                 "attn_merge"]
 
 c_p = ctypes.c_void_p

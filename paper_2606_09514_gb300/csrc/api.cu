@@ -54,7 +54,7 @@ static void free_ctx(buddy_ctx* x) {
   for (cudaEvent_t e : c.ev_pool) cudaEventDestroy(e);
   void* ptrs[] = {c.rope_cos, c.rope_sin, c.status, c.xn, c.act, c.attn_out, c.qkv, c.q,
                   c.attn_m, c.attn_l, c.attn_acc, c.attn_ctr, c.dm_u, c.mask, c.sel, c.scores, c.rows,
-                  c.count, c.h_in_stage, c.h_out_stage, c.k_stage, c.mask_stage, c.xn_lo, c.act_lo, c.attn_lo, c.lk_bar,
+                  c.count, c.h_in_stage, c.h_out_stage, c.k_stage, c.mask_stage, c.xn_lo, c.act_lo, c.attn_lo,
                   c.gemm_ws, c.gemm_ctr, c.attn_meta};
   for (void* p : ptrs)
     if (p) cudaFree(p);
@@ -105,10 +105,6 @@ extern "C" int buddy_create(const buddy_config* cfg, buddy_ctx** out) {
   c.qd = c.nq * c.hd; c.kvd = c.nkv * c.hd; c.qkvN = c.qd + 2 * c.kvd;
   c.maxB = g.max_batch; c.max_pos = g.max_pos; c.dtype = g.dtype;
   c.esz = g.dtype == BUDDY_DTYPE_BF16 ? 2 : 4;
-  {
-    const char* env = getenv("BUDDY_PDL");
-    c.pdl = !(env && env[0] == '0');
-  }
   auto fail = [&](cudaError_t e) {
     fprintf(stderr, "libbuddy: create: %s\n", cudaGetErrorString(e));
     free_ctx(x);
@@ -253,7 +249,7 @@ extern "C" int buddy_set_profiling(buddy_ctx* ctx, int32_t on) {
 extern "C" const char* buddy_profile_class_name(int32_t cls) {
   static const char* names[BUDDY_PROF_NCLASS] = {"check", "rmsnorm", "gemm_qkv", "qkv_finalize",
                                                  "attention", "gemm_o", "gemm_gate_up", "gemm_down",
-                                                 "route", "compact", "other", "layer", "gemm_fixup",
+                                                 "route", "compact", "other", "gemm_fixup",
                                                  "attn_merge"};
   return (cls >= 0 && cls < BUDDY_PROF_NCLASS) ? names[cls] : "unknown";
 }
@@ -307,10 +303,6 @@ static void run_gemm(Ctx& c, int epi, GemmArgs a, int layer, int which, cudaStre
 // from `src` and the output goes to `H`.
 static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, const float* src,
                           float* H, cudaStream_t s, bool prof) {
-  if (c.use_lk) {
-    ProfScope p(c, s, BUDDY_PROF_LAYER, 1, prof);
-    if (launch_layer_kernel(c, kv, l, sel, src, H, s)) return;
-  }
   const buddy_layer_weights& W = c.layers[l];
   // The first layer feeds the router: its GEMM inputs are kept as bf16 hi + lo
   // pairs so that its output is a continuous function of the inputs.

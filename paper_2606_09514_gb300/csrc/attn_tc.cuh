@@ -45,19 +45,10 @@
 
 namespace buddy {
 
-#ifndef BUDDY_TCA_CHUNK
-#define BUDDY_TCA_CHUNK 32
-#endif
-constexpr int kTcaChunk = BUDDY_TCA_CHUNK;   // positions per warp chunk (16 or 32)
-#ifndef BUDDY_TCA_WARPS
-#define BUDDY_TCA_WARPS 4
-#endif
-constexpr int kTcaWarps = BUDDY_TCA_WARPS;
+constexpr int kTcaChunk = 32;     // positions per warp chunk (16 or 32)
+constexpr int kTcaWarps = 4;
 constexpr int kTcaThreads = 32 * kTcaWarps;
-#ifndef BUDDY_TCA_STAGES
-#define BUDDY_TCA_STAGES 3
-#endif
-constexpr int kTcaStages = BUDDY_TCA_STAGES;   // chunk buffers per warp (kTcaStages - 1 in flight)
+constexpr int kTcaStages = 3;     // chunk buffers per warp (kTcaStages - 1 in flight)
 constexpr int kTcaMinShare = 2 * kTcaChunk;   // positions of a warp's share, at least
 constexpr int kTcaMergeThreads = 256;         // merge kernel: one CTA per stream
 constexpr int kTcaWarpMerge = 4;              // streams of at most this many spans merge in the kernel

@@ -1,5 +1,4 @@
-// Building blocks of the tensor-core decode GEMM, shared by the GEMM kernel
-// (gemm_tc.cu) and the per-layer persistent kernel (layer_kernel.cu).
+// Building blocks of the tensor-core decode GEMM (gemm_tc.cu).
 //
 //   C[j][n] = sum_k X[j][k] * W[n][k]      (j < m active rows, n < N features)
 //
@@ -21,9 +20,7 @@
 //
 // The accumulator of a unit (tile, K split) is mt x 256 fp32 TMEM columns.
 // The ring fills shared memory and, with one M-tile, two accumulators let the
-// MMAs of the next unit overlap the epilogue.  (BUDDY_TC_DUAL=1 instead gives
-// small batches a short ring and one accumulator so that two GEMM CTAs fit on
-// an SM; measured slower, kept opt-in.)
+// MMAs of the next unit overlap the epilogue.
 //
 // Panel mode (up to 8 rows): the ring holds weight tiles only and the
 // activations of the QKV and gate/up GEMMs are the RMSNorm of the fp32

@@ -372,10 +372,10 @@ static int choose_splits(int tiles, int kb, int sms) {
   return best_eff > 0 ? best : fb;
 }
 
+// bf16 shapes always take the tensor-core path: sm_103 and at most 256 rows
+// (buddy_create rejects anything else).
 bool gemm_tc_supported(const Ctx& c) {
   if (c.dtype != BUDDY_DTYPE_BF16 || c.maxB > 256 || (c.hd != 64 && c.hd != 128)) return false;
-  const char* env = getenv("BUDDY_GEMM");
-  if (env && env[0] == 's') return false;   // "simt": CUDA-core kernel for every GEMM
   int major = 0, minor = 0;
   cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, c.device);
   cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, c.device);
@@ -383,25 +383,18 @@ bool gemm_tc_supported(const Ctx& c) {
 }
 
 int gemm_tc_prepare(Ctx& c) {
-  c.use_tc = gemm_tc_supported(c);
-  c.use_lk = false;
+  c.use_tc = c.dtype == BUDDY_DTYPE_BF16;
   if (!c.use_tc) return BUDDY_OK;
+  if (!gemm_tc_supported(c)) return BUDDY_ERR_ARG;
   // geometry: 256 weight rows per tile; one M-tile per 128 rows of the batch
   c.tc_bw = kTileN;
   c.tc_mt = c.maxB > 128 ? 2 : 1;
   c.tc_rows_max = std::max(16, (c.maxB + 15) & ~15);
   c.tc_xr = c.tc_mt == 1 ? (uint32_t)c.tc_rows_max * 128u : kXTileMax;
-  // One CTA per SM with the full ring; optionally (BUDDY_TC_DUAL=1) two CTAs
-  // per SM with a short ring and one accumulator, where at least two stages
-  // fit in half of the shared memory (measured slower on the 8B decode chain).
-  const int full_limit = 227 * 1024 - 2 * 1024;   // room for static shared memory
-  const int half_limit = 111 * 1024;
-  const uint32_t sb_max = (uint32_t)c.tc_bw * 128u + 2u * c.tc_mt * c.tc_xr;
-  const char* dual_env = getenv("BUDDY_TC_DUAL");
-  c.tc_dual = dual_env && dual_env[0] == '1' && (int)((half_limit - 1024) / sb_max) >= 2;
-  c.tc_acc_bufs = c.tc_dual || c.tc_mt == 2 ? 1 : 2;
-  c.tc_tmem_cols = c.tc_dual ? 256 : 512;
-  const int limit = c.tc_dual ? half_limit : full_limit;
+  // One CTA per SM with the full ring.
+  const int limit = 227 * 1024 - 2 * 1024;   // room for static shared memory
+  c.tc_acc_bufs = c.tc_mt == 2 ? 1 : 2;
+  c.tc_tmem_cols = 512;
   for (int v = 0; v < 2; ++v) {
     const uint32_t stage_bytes = (uint32_t)c.tc_bw * 128u + (uint32_t)(v + 1) * c.tc_mt * c.tc_xr;
     c.tc_stages[v] = std::min(kTcMaxStages, (int)((limit - 1024) / stage_bytes));
@@ -471,18 +464,8 @@ int gemm_tc_prepare(Ctx& c) {
   }
   // Above kTcDeferRows rows a tile's partials are too many for the one CTA
   // that would finish it (m x 256 fp32 per split): a fixup kernel spreads
-  // them over all SMs.  BUDDY_TC_DEFER_ROWS overrides the threshold.
-  {
-    const char* env = getenv("BUDDY_TC_DEFER_ROWS");
-    const int thr = env && env[0] ? atoi(env) : kTcDeferRows;
-    c.tc_defer = c.maxB > thr;
-  }
-  const char* lk_env = getenv("BUDDY_LAYER_KERNEL");
-  c.use_lk = layer_kernel_supported(c) && lk_env && lk_env[0] == '1';   // opt-in
-  if (c.use_lk && !c.lk_bar) {
-    if (cudaMalloc(&c.lk_bar, 2 * sizeof(unsigned)) != cudaSuccess) return BUDDY_ERR_CUDA;
-    if (cudaMemset(c.lk_bar, 0, 2 * sizeof(unsigned)) != cudaSuccess) return BUDDY_ERR_CUDA;
-  }
+  // them over all SMs.
+  c.tc_defer = c.maxB > kTcDeferRows;
   const cudaFuncAttribute A = cudaFuncAttributeMaxDynamicSharedMemorySize;
   const int qs0 = std::max(c.tc_smem[0], c.tc_panel ? c.tc_psmem[0] : 0);
   const int qs1 = std::max(c.tc_smem[1], c.tc_panel ? c.tc_psmem[1] : 0);

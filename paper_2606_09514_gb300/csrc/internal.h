@@ -117,10 +117,6 @@ void launch_pool_refresh(const Ctx& c, const buddy_kv_state& kv, int n_seq, cons
 // GEMMs (gemm_simt.cu, gemm_tc.cu)
 void launch_gemm_simt(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s);
 bool gemm_tc_supported(const Ctx& c);
-// layer_kernel.cu: one executed block as one persistent cooperative kernel
-bool layer_kernel_supported(const Ctx& c);
-bool launch_layer_kernel(const Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, const float* src, float* H,
-                         cudaStream_t s);
 void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s);
 void launch_gemm_fix(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s);   // with c.tc_defer
 
@@ -174,10 +170,7 @@ struct Ctx {
   int tc_bw = 256, tc_mt = 1, tc_rows_max = 16, tc_acc_bufs = 2;   // tile geometry (gemm_common.cuh)
   int tc_stages[2] = {1, 1}, tc_smem[2] = {0, 0};                   // [plain, split activations]
   uint32_t tc_stage_bytes[2] = {0, 0}, tc_w_off[2] = {0, 0}, tc_xr = 0, tc_tmem_cols = 512;
-  bool tc_dual = false;                   // two GEMM CTAs per SM (short ring, one accumulator)
   int tc_splits[4] = {1, 1, 1, 1}, tc_tiles[4] = {1, 1, 1, 1};
-  bool use_lk = false;                    // per-layer persistent kernel (small batches)
-  unsigned* lk_bar = nullptr;             // its grid barrier [arrivals, generation]
   float* gemm_ws = nullptr;
   size_t gemm_ws_elems = 0;
   int32_t* gemm_ctr = nullptr;

@@ -263,41 +263,3 @@ def test_generator_identical_on_cpu_and_gpu():
         a = synth.normal((n,), key, 1.0, torch.float32, "cpu", start=start)
         b = synth.normal((n,), key, 1.0, torch.float32, "cuda", start=start).cpu()
         assert torch.equal(a.view(torch.int32), b.view(torch.int32))
-
-
-# With BUDDY_LAYER_KERNEL=1, small batches (at most 16 rows, head_dim 128) run
-# each block as one persistent kernel; these exercise that path against the
-# oracle.
-T_QWEN_B12 = C.scaled(C.T_QWEN, ctx=[0, 1, 63, 64, 65, 127, 128, 129, 700, 17, 256, 1000],
-                      k=[1, 5, 3, 2, 4, 5, 1, 1, 2, 3, 4, 5], name="t-qwen-bf16-b12")
-
-
-def test_decode_parity_layer_kernel(monkeypatch):
-    monkeypatch.setenv("BUDDY_LAYER_KERNEL", "1")
-    worst, _ = run_parity(T_QWEN_B12)
-    assert worst < 2e-2
-
-
-def test_decode_parity_layer_kernel_graph_prior(monkeypatch):
-    monkeypatch.setenv("BUDDY_LAYER_KERNEL", "1")
-    run_parity(T_QWEN_B12, steps=2, use_graph=True, prior=True)
-
-
-def test_layer_kernel_matches_separate_kernels(monkeypatch):
-    """The persistent per-layer kernel and the separate kernels compute the
-    same block (they may differ in reduction order only)."""
-    outs = []
-    for lk in ("1", "0"):
-        monkeypatch.setenv("BUDDY_LAYER_KERNEL", lk)
-        dw = D.build(T_QWEN_B12)
-        h_out = torch.empty(T_QWEN_B12.batch, T_QWEN_B12.shape.d_model, device="cuda")
-        mask = torch.empty(T_QWEN_B12.batch, T_QWEN_B12.shape.n_layers, dtype=torch.uint8, device="cuda")
-        for t in range(2):
-            dw.ctx.buddy_decode_step(dw.kv, synth.workload_h_in(T_QWEN_B12, t, "cuda"), dw.k, h_out, mask)
-        torch.cuda.synchronize()
-        assert dw.ctx.buddy_device_status() == 0
-        outs.append((h_out.cpu().numpy(), mask.cpu().numpy()))
-        dw.ctx.close()
-    np.testing.assert_array_equal(outs[0][1], outs[1][1])
-    for i in range(T_QWEN_B12.batch):
-        assert P.max_rel_err(outs[0][0][i], outs[1][0][i]) < 2e-2

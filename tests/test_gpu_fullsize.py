@@ -1,24 +1,30 @@
-"""GPU parity at the benchmark workloads' full sizes, in the launch configuration
-bench.py times (CUDA graph, programmatic dependent launch).
+"""GPU parity at the benchmark workloads' full sizes and their own step counts,
+in the launch configuration bench.py times (CUDA graph, programmatic
+dependent launch).
 
-One decode step per workload.  The oracle evaluates the first layer and the
-router for every sequence (routes checked with the near-tie rule, compaction
-bit-exact for every layer) and the full routed depth for a few sampled
-sequences (hidden state and the K/V written at the new position), streaming
-their caches one layer at a time.
+Every workload runs its decode trajectory on the GPU (Llama-3-8B B=1: 64
+steps, B=64 mixed: 32, Llama-2-13B B=32: 32, Qwen2.5-7B B=256: 16), free
+running: each step's new K/V feed the next.  The oracle evaluates the same
+trajectory on its own state (tests/trajectory.py, one block at a time):
+
+  * layers 0..c and the router for every sequence at every step: routes are
+    checked with the near-tie rule and the row compaction bit-exactly, for
+    every sequence and step;
+  * the routed layers for a few sampled sequences: the hidden state after the
+    last layer and the K/V written at every layer, at every step.
 """
 import numpy as np
 import pytest
 import torch
 
 import parity as P
+import trajectory as T
 from oracle import adapter as A
-from oracle import buddy_oracle as O
 from workloads import configs as C
 from workloads import device as D
 from workloads import synth
 
-pytestmark = [pytest.mark.gpu, pytest.mark.slow]
+pytestmark = pytest.mark.gpu
 
 CASES = [
     (C.C2_LLAMA3_B1, [0]),
@@ -28,58 +34,75 @@ CASES = [
 ]
 
 
-@pytest.mark.parametrize("w,sampled", CASES, ids=[c[0].name for c in CASES])
-def test_fullsize_step_parity(w, sampled):
+def run_gpu_trajectory(w, sampled, dev="cuda"):
+    """Decode w.steps steps on the GPU; record the routing outputs of every
+    sequence and, for the sampled ones, the final hidden state and the K/V
+    written at every layer."""
     s = w.shape
-    dev = "cuda"
+    B, L = w.batch, s.n_layers
     dw = D.build(w, extra_steps=2, use_graph=True)
-    B, L, Lm = w.batch, s.n_layers, s.l_mid
-    h_in = synth.workload_h_in(w, 0, dev)
+    n0 = w.contexts()
     h_out = torch.empty(B, s.d_model, device=dev)
     mask = torch.empty(B, L, dtype=torch.uint8, device=dev)
     rows = torch.empty(L, B, dtype=torch.int32, device=dev)
     count = torch.empty(L, dtype=torch.int32, device=dev)
-    scores = torch.empty(B, Lm, device=dev)
-    dw.ctx.buddy_decode_step(dw.kv, h_in, dw.k, h_out, mask, rows, count, scores)
-    torch.cuda.synchronize()
-    assert dw.ctx.buddy_device_status() == 0
-    g_mask = mask.cpu().numpy()
-    g_sel = P.sel_from_mask(g_mask)
-    # K/V the GPU wrote at the new position, for the sampled sequences
-    n0 = w.contexts()
-    g_kv = {(l, i): (dw.kv.view("k", l, i)[:, int(n0[i]), :].float().cpu().numpy(),
-                     dw.kv.view("v", l, i)[:, int(n0[i]), :].float().cpu().numpy())
-            for l in range(L) for i in sampled}
-    g_h = h_out.cpu().numpy()
-    g_scores = scores.cpu().numpy()
-    g_rows, g_count = rows.cpu().numpy(), count.cpu().numpy()
+    scores = torch.empty(B, s.n_cand, device=dev)
+    rec = []
+    for t in range(w.steps):
+        h_in = synth.workload_h_in(w, t, dev)
+        dw.ctx.buddy_decode_step(dw.kv, h_in, dw.k, h_out, mask, rows, count, scores)
+        torch.cuda.synchronize()
+        assert dw.ctx.buddy_device_status() == 0, t
+        kv = {}
+        for i in sampled:
+            p = int(n0[i]) + t
+            kv[i] = (torch.stack([dw.kv.view("k", l, i)[:, p, :] for l in range(L)]).float().cpu().numpy(),
+                     torch.stack([dw.kv.view("v", l, i)[:, p, :] for l in range(L)]).float().cpu().numpy())
+        rec.append(dict(mask=mask.cpu().numpy(), rows=rows.cpu().numpy(), count=count.cpu().numpy(),
+                        scores=scores.cpu().numpy(), h={i: h_out[i].cpu().numpy() for i in sampled}, kv=kv))
+    np.testing.assert_array_equal(dw.kv.len.cpu().numpy(), n0 + w.steps)
     dw.ctx.close()
     del dw
     torch.cuda.empty_cache()
+    return rec
 
+
+@pytest.mark.parametrize("w,sampled", CASES, ids=[c[0].name for c in CASES])
+def test_fullsize_trajectory_parity(w, sampled):
+    s = w.shape
+    dev = "cuda"
+    L, S = s.n_layers, w.steps
+    rec = run_gpu_trajectory(w, sampled, dev)
     model = A.build_model(s, w.seed, layer_source=lambda l: synth.layer_weights(s, w.seed, l, dev),
                           dm_source=lambda: synth.dm_weights(s, w.seed, dev), cache_layers=1)
-    st = A.lazy_state(s, w.seed, n0, gen_device=dev)
-    k = w.budgets()
-    route = O.first_layer_and_route(model, st, A.to_f64(h_in), k)
-    st.drop(0)
-    sel, fails, adopted = P.adopt_routes(route.scores, route.sel, g_sel, k)
-    assert not fails, fails[:5]
-    route.sel = sel
-    np.testing.assert_allclose(g_scores, route.scores, rtol=0, atol=P.ROUTE_MARGIN / 4)
-    np.testing.assert_array_equal(g_mask.sum(1), k + 2)
-    res = O.routed_layers(model, st, route, seqs=sampled)
-    for l in range(L):
-        assert g_count[l] == len(res.rows[l]), l
-        assert g_rows[l, : g_count[l]].tolist() == res.rows[l], l
-    for i in sampled:
-        e = P.max_rel_err(g_h[i], res.h_out[i])
-        print(f"{w.name}: sequence {i} hidden max rel err {e:.3e}; adopted near-ties {adopted}")
-        assert e < P.HIDDEN_TOL[s.dtype], (i, e)
+    n0, k = w.contexts(), w.budgets()
+    h_in = [A.to_f64(synth.workload_h_in(w, t, dev)) for t in range(S)]
+    ev = T.evaluate(model, n0, k, h_in, sampled,
+                    lambda layers, seqs: A.build_state(s, w.seed, n0, layers=layers, seqs=seqs, gen_device=dev),
+                    gpu_masks=[r["mask"] for r in rec])
+    assert not ev["fails"], ev["fails"][:5]
+    first = model.shape.first_candidate
+    for t in range(S):
+        g = rec[t]
+        np.testing.assert_allclose(g["scores"], ev["scores"][t], rtol=0, atol=P.ROUTE_MARGIN / 4)
+        np.testing.assert_array_equal(g["mask"].sum(1), np.asarray(ev["k"][t]) + 1 + first)
+        rows = T.O.compaction(ev["sel"][t], L, first)
         for l in range(L):
-            gk, gv = g_kv[(l, i)]
-            ok, ov = res.kv_new[(l, i)]
-            if g_mask[i, l]:
-                assert P.max_rel_err(gk, ok) < P.KV_TOL[s.dtype] and P.max_rel_err(gv, ov) < P.KV_TOL[s.dtype], (l, i)
-            else:
-                assert not gk.any() and not gv.any(), (l, i)
+            assert g["count"][l] == len(rows[l]), (t, l)
+            assert g["rows"][l, : g["count"][l]].tolist() == rows[l], (t, l)
+    worst = kv_err = 0.0
+    for i in sampled:
+        for t in range(S):
+            e = P.max_rel_err(rec[t]["h"][i], ev["H"][i][t])
+            worst = max(worst, e)
+            assert e < P.HIDDEN_TOL[s.dtype], (i, t, e)
+            for l in range(L):
+                gk, gv = rec[t]["kv"][i][0][l], rec[t]["kv"][i][1][l]
+                o = ev["kv"][(l, i)][t]
+                if o is not None and o[0].any():
+                    kv_err = max(kv_err, P.max_rel_err(gk, o[0]), P.max_rel_err(gv, o[1]))
+                else:
+                    assert not gk.any() and not gv.any(), (l, i, t)
+    print(f"{w.name}: {S} steps, sampled {sampled}: worst hidden max rel err {worst:.3e}, "
+          f"worst K/V {kv_err:.3e}, adopted near-ties {ev['adopted']}")
+    assert kv_err < P.KV_TOL[s.dtype]

@@ -55,6 +55,34 @@ def test_noalloc_router_matches_context_router_twice():
         np.testing.assert_array_equal(m1, m0)
         np.testing.assert_array_equal(m1.sum(1), k.cpu().numpy() + 2)
 
+    # a budget outside [1, L-2] (seen only by the device): the flags word says
+    # so, nothing else is written, and the next valid call is not held up by
+    # the abort word this call left in the shared scratch
+    bad = dw.k.clone()
+    bad[4] = 0
+    sel = torch.full((Bn, Lm), -7, dtype=torch.int32, device=dev)
+    mask = torch.full((Bn, L), 9, dtype=torch.uint8, device=dev)
+    sc = torch.full((Bn, Lm), 123.0, device=dev)
+    flags = torch.full((1,), -1, dtype=torch.int32, device=dev)
+    h1 = synth.h_in(s, 77, 0, range(Bn), dev)
+    pkg.binding.buddy_route_noalloc(s, dw.dm, dw.kv.pool_sum, dw.kv.len, h1, bad, sel, mask, sc, flags,
+                                    prior=dw.prior, omega=0.1)
+    torch.cuda.synchronize()
+    assert int(flags.item()) == B.BUDDY_DEV_BAD_BUDGET
+    assert torch.all(sel == -7) and torch.all(mask == 9) and torch.all(sc == 123.0)
+    flags.fill_(-1)
+    pkg.binding.buddy_route_noalloc(s, dw.dm, dw.kv.pool_sum, dw.kv.len, h1, dw.k, sel, mask, sc, flags,
+                                    prior=dw.prior, omega=0.1)
+    sel2 = torch.empty_like(sel)
+    mask2 = torch.empty_like(mask)
+    sc2 = torch.empty_like(sc)
+    dw.ctx.buddy_route(dw.kv, h1, dw.k, sel2, mask2, sc2)
+    torch.cuda.synchronize()
+    assert int(flags.item()) == 0
+    np.testing.assert_array_equal(sel.cpu().numpy(), sel2.cpu().numpy())
+    np.testing.assert_array_equal(mask.cpu().numpy(), mask2.cpu().numpy())
+    np.testing.assert_allclose(sc.cpu().numpy(), sc2.cpu().numpy(), rtol=0, atol=P.ROUTE_MARGIN / 4)
+
     # sizes beyond the static scratch are rejected before any launch
     big = torch.zeros(300, s.d_model, device=dev)
     lib = B.load_library()
