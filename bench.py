@@ -4,7 +4,10 @@ python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                 [--workload NAME] [--no-graph]
 
 Default workload: Llama-3-8B shape, bf16, batch 1, context 2048, budget k = 15
-of 30 middle layers (the configuration the headline metric is quoted on).
+of 30 middle layers (the configuration the headline metric is quoted on).  The
+default run also times the other bf16 workloads (Llama-3-8B B=64 mixed
+budgets, Llama-2-13B B=32, Qwen2.5-7B B=256), each over its own step count,
+and reports them under "per_config".
 A step = one budget-routed decode step of the whole batch (layer 0, router,
 compaction, the selected middle layers on their sub-batches, last layer).
 Inputs (weights 14 GB, KV cache) are resident in HBM and larger than L2.
@@ -33,7 +36,9 @@ METRIC = "budget-routed decode tokens/s at 1 GB300 per budget; % of HBM/tensor r
 # ncu dram bytes (read + write) per launch of the dominant kernel, from the
 # committed ncu summary of the gate/up GEMM (3-layer model with the same layer
 # shapes as the 32-layer bench workload); absent for kernels not captured
-NCU_TRAFFIC_PER_LAUNCH = {"gemm_gate_up": 238353664}
+NCU_TRAFFIC_PER_LAUNCH = {("llama3-8b-b1", "gemm_gate_up"): 238353664}
+DEFAULT_WORKLOAD = "llama3-8b-b1"
+PER_CONFIG = ["llama3-8b-b64-mixed", "llama2-13b-b32", "qwen2.5-7b-b256"]
 
 
 def _peaks():
@@ -209,27 +214,25 @@ def class_bytes(s, masks, ctxs, B):
 # ---------------------------------------------------------------------------
 # Our arm
 # ---------------------------------------------------------------------------
-def run_ours(args, ws, rank, local):
+NOMINAL_HBM_GBS = 7900.0   # GB300 HBM3e, nominal (context for the measured-peak fractions)
+
+
+def measure(w, K, W, dev, ws, local, use_graph=True, e2e=True):
+    """Times K budget-routed decode steps of workload w (after W warm-up
+    steps) on device `dev`, then profiles kernel classes over a few more
+    direct-launch steps and (optionally) times the host-buffer entry point."""
     import torch
 
-    from workloads import configs as C
     from workloads import cost
     from workloads import device as D
     from workloads import synth
 
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    if ws > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=dev)
-    w = C.BY_NAME[args.workload]
     s = w.shape
     B = w.batch
-    K, W = args.steps, args.warmup
     prof_steps = min(K, 8)
-    e2e_steps = K
+    e2e_steps = K if e2e else 0
     extra = W + K + prof_steps + e2e_steps + 2
-    dw = D.build(w, device=dev, extra_steps=extra, use_graph=not args.no_graph)
+    dw = D.build(w, device=dev, extra_steps=extra, use_graph=use_graph)
     ctx, kv = dw.ctx, dw.kv
     n_steps_total = W + K + prof_steps + e2e_steps
     h_all = [synth.h_in(s, w.seed, t, range(B), dev) for t in range(n_steps_total)]
@@ -252,13 +255,10 @@ def run_ours(args, ws, rank, local):
         raise RuntimeError("device error flag during warm-up")
 
     # timed region: K steps, positions advancing
-    n_ctx_timed = []
-    masks = []
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clk:
         _barrier(ws)
         torch.cuda.synchronize(dev)
-        lens0 = kv.len.cpu().numpy().copy()
         start.record(stream)
         for t in range(K):
             h_buf.copy_(h_all[step], non_blocking=True)
@@ -286,22 +286,26 @@ def run_ours(args, ws, rank, local):
         step += 1
     prof = ctx.buddy_profile_read()
     ctx.buddy_set_profiling(False)
-    ctx.buddy_set_options(not args.no_graph)
+    ctx.buddy_set_options(use_graph)
 
-    # end to end through the host-buffer entry point (pinned buffers)
-    h_host = [h.cpu().pin_memory() for h in h_all[step:step + e2e_steps]]
-    k_host = dw.k.cpu().pin_memory()
-    o_host = torch.empty(B, s.d_model).pin_memory()
-    m_host = torch.empty(B, s.n_layers, dtype=torch.uint8).pin_memory()
-    ctx.buddy_decode_step_host(kv, h_host[0], k_host, o_host, m_host)   # graph for the staging buffers
-    step += 1
-    _barrier(ws)
-    t0 = time.perf_counter()
-    for t in range(1, e2e_steps):
-        ctx.buddy_decode_step_host(kv, h_host[t], k_host, o_host, m_host)
-    e2e_s = time.perf_counter() - t0
-    e2e_s = _max_over_ranks(e2e_s, ws, dev)
-    e2e_n = e2e_steps - 1
+    e2e_out = None
+    if e2e:
+        # end to end through the host-buffer entry point (pinned buffers)
+        h_host = [h.cpu().pin_memory() for h in h_all[step:step + e2e_steps]]
+        k_host = dw.k.cpu().pin_memory()
+        o_host = torch.empty(B, s.d_model).pin_memory()
+        m_host = torch.empty(B, s.n_layers, dtype=torch.uint8).pin_memory()
+        ctx.buddy_decode_step_host(kv, h_host[0], k_host, o_host, m_host)   # graph for the staging buffers
+        step += 1
+        _barrier(ws)
+        t0 = time.perf_counter()
+        for t in range(1, e2e_steps):
+            ctx.buddy_decode_step_host(kv, h_host[t], k_host, o_host, m_host)
+        e2e_s = time.perf_counter() - t0
+        e2e_s = _max_over_ranks(e2e_s, ws, dev)
+        e2e_out = {"value": round(ws * B * (e2e_steps - 1) / e2e_s, 2), "unit": "tokens/s",
+                   "h2d_bytes_per_step": B * s.d_model * 4 + B * 4,
+                   "d2h_bytes_per_step": B * s.d_model * 4 + B * s.n_layers}
 
     # algorithmic cost of the profiled steps (realised masks and lengths)
     hbm, tflops, peak_src = _peaks()
@@ -310,7 +314,6 @@ def run_ours(args, ws, rank, local):
         c = cost.step_cost(s, m_, n_[:B])
         for key in c_sum:
             c_sum[key] += c[key]
-    prof_ms_total = sum(v[0] for v in prof.values())
     # dominant kernel class and its algorithmic bytes (summed over the profiled steps)
     dom = max(prof, key=lambda k: prof[k][0])
     per_class_bytes = class_bytes(s, prof_masks, prof_ctx, B)
@@ -321,14 +324,17 @@ def run_ours(args, ws, rank, local):
         avg_s = prof[dom][0] / 1e3 / launches
         ach = bytes_per_launch / avg_s / 1e9
         roof = {"bound": "hbm", "kernel": dom, "achieved": round(ach, 1), "peak": hbm, "unit": "GB/s",
-                "frac": round(ach / hbm, 4), "traffic": NCU_TRAFFIC_PER_LAUNCH.get(dom),
+                "frac": round(ach / hbm, 4), "traffic": NCU_TRAFFIC_PER_LAUNCH.get((w.name, dom)),
                 "bytes_per_launch": int(bytes_per_launch), "avg_launch_us": round(avg_s * 1e6, 2),
-                "launches": launches, "peak_source": f"{peak_src} hbm_gbs"}
+                "launches": launches, "peak_source": f"{peak_src} hbm_gbs",
+                "frac_of_nominal": round(ach / NOMINAL_HBM_GBS, 4)}
     t_roof = max(c_sum["bytes"] / (hbm * 1e9), c_sum["flops"] / (tflops * 1e12)) / prof_steps
-    step_s = ms_max / 1e3 / K
-    route_frac = (prof["route"][0] + prof["compact"][0]) / max(prof_ms_total, 1e-9)
+    t_roof_nom = max(c_sum["bytes"] / (NOMINAL_HBM_GBS * 1e9), c_sum["flops"] / (tflops * 1e12)) / prof_steps
+    step_ms = ms_max / K
+    # router + compaction per step (direct-launch events) over the graph step time
+    route_ms = (prof["route"][0] + prof["compact"][0]) / prof_steps
     launches_per_step = sum(v[1] for v in prof.values()) / prof_steps
-    # the timed steps launch every middle layer (a layer no row selected exits
+    # the timed steps launch every routed layer (a layer no row selected exits
     # at once); the profiled steps launch only the selected ones
     per_layer = ("rmsnorm", "gemm_qkv", "qkv_finalize", "attention", "gemm_o", "gemm_gate_up", "gemm_down",
                  "gemm_fixup", "attn_merge")
@@ -336,28 +342,59 @@ def run_ours(args, ws, rank, local):
     per_layer_kernels = sum(prof.get(k, (0, 0))[1] for k in per_layer) / max(exec_layers * prof_steps, 1)
     graph_extra = max(s.n_layers - exec_layers, 0) * per_layer_kernels
     out = {
-        "metric": METRIC, "value": round(value, 2), "unit": "tokens/s", "n_gpus": ws, "steps": K,
-        "warmup": W, "ms_per_step": round(ms_max / K, 4), "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": s.dtype, "data": "synthetic (seeded counter-based generator)",
+        "value": round(value, 2), "unit": "tokens/s", "ms_per_step": round(step_ms, 4), "steps": K,
+        "warmup": W, "dtype": s.dtype,
         "config": {"workload": w.name, "model": s.name, "batch": B, "ctx": w.ctx_args,
-                   "k": w.k_args, "layers": s.n_layers, "parallelism": f"replicas x{ws}",
-                   "graph": not args.no_graph,
-                   "l2": "inputs larger than L2 (per-step weight stream %.1f GB)" % (c_sum["weight_bytes"] / prof_steps / 1e9)},
+                   "k": w.k_args, "layers": s.n_layers, "parallelism": f"replicas x{ws}", "graph": use_graph,
+                   "l2": "inputs larger than L2 (per-step weight stream %.1f GB)"
+                         % (c_sum["weight_bytes"] / prof_steps / 1e9)},
+        "paths": ctx.buddy_get_paths(),
         "roofline": roof,
-        "step_roofline": {"t_roof_ms": round(t_roof * 1e3, 4), "frac": round(t_roof / step_s, 4),
+        "step_roofline": {"t_roof_ms": round(t_roof * 1e3, 4), "frac": round(t_roof * 1e3 / step_ms, 4),
+                          "frac_of_nominal_hbm": round(t_roof_nom * 1e3 / step_ms, 4),
                           "bytes_per_step": int(c_sum["bytes"] / prof_steps),
                           "flops_per_step": int(c_sum["flops"] / prof_steps), "peak_gbs": hbm,
-                          "peak_source": peak_src},
-        "route_compact_frac": round(route_frac, 4),
-        "kernel_ms_per_step": {k: round(v[0] / prof_steps, 4) for k, v in prof.items()},
+                          "nominal_gbs": NOMINAL_HBM_GBS, "peak_source": peak_src},
+        "route_compact_ms_per_step": round(route_ms, 4),
+        "route_compact_frac": round(route_ms / step_ms, 4),
+        "kernel_ms_per_step": {k: round(v[0] / prof_steps, 4) for k, v in prof.items() if v[1] > 0},
         "kernel_gbs": {k: round(per_class_bytes[k] / (prof[k][0] / 1e3) / 1e9, 1)
                        for k in per_class_bytes if prof[k][0] > 0},
-        "e2e": {"value": round(ws * B * e2e_n / e2e_s, 2), "unit": "tokens/s",
-                "h2d_bytes_per_step": B * s.d_model * 4 + B * 4,
-                "d2h_bytes_per_step": B * s.d_model * 4 + B * s.n_layers},
+        "e2e": e2e_out,
         "gpu_launches": int(round((launches_per_step + graph_extra) * K)),
         "clocks": clk.summary(),
     }
+    ctx.close()
+    del dw, kv, ctx, h_all
+    torch.cuda.empty_cache()
+    return out
+
+
+def run_ours(args, ws, rank, local):
+    import torch
+
+    from workloads import configs as C
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    w = C.BY_NAME[args.workload]
+    head = measure(w, args.steps, args.warmup, dev, ws, local, use_graph=not args.no_graph)
+    out = {"metric": METRIC, "value": head["value"], "unit": "tokens/s", "n_gpus": ws, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": head["ms_per_step"], "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": head["dtype"],
+           "data": "synthetic (seeded counter-based generator)"}
+    out.update({k: v for k, v in head.items() if k not in ("value", "unit", "ms_per_step", "steps", "warmup",
+                                                           "dtype")})
+    if args.workload == DEFAULT_WORKLOAD and not args.headline_only:
+        # the other bf16 workloads, each over its own step count, on the same box
+        out["per_config"] = {}
+        for name in PER_CONFIG:
+            wc = C.BY_NAME[name]
+            r = measure(wc, wc.steps, args.warmup, dev, ws, local, use_graph=not args.no_graph, e2e=False)
+            out["per_config"][name] = r
     if rank == 0 and not args.no_cpu:
         o = oracle_sample(w, n_layers_sample=None, steps=1, device=dev)
         out["cpu_baseline"] = {"value": round(o["tokens"] / o["scaled_seconds"], 5), "unit": "tokens/s",
@@ -366,7 +403,6 @@ def run_ours(args, ws, rank, local):
                                          f"weight generation and host copy excluded)"}
     if rank == 0:
         print(json.dumps(out), flush=True)
-    ctx.close()
     if ws > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
@@ -403,7 +439,8 @@ def main():
     ap.add_argument("--steps", type=int, default=64)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="llama3-8b-b1")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--headline-only", action="store_true", help="skip the per_config workloads")
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline oracle sample")
     args = ap.parse_args()

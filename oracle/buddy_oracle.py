@@ -421,6 +421,7 @@ class RouteResult:
     k: List[int]                   # budget used per sequence (given or predicted)
     sel: List[List[int]]           # per sequence, ascending executed routed layers
     kv_new: Dict[tuple, tuple]     # (layer <= c, seq) -> (k_t, v_t) written
+    x: Optional[np.ndarray] = None  # [B, 2d] router inputs
 
 
 @dataclasses.dataclass
@@ -460,7 +461,7 @@ def first_layers_and_route(model: Model, st: KVState, h_in: np.ndarray, k: Seque
         for i in range(B):
             kv_new[(l, i)] = (kn[i], vn[i])
     scores = np.empty((B, sh.n_cand))
-    ks, sel = [], []
+    ks, sel, xs = [], [], []
     for i in range(B):
         K, V = st.get(c, i)
         kt, vt = kv_new[(c, i)]
@@ -468,7 +469,8 @@ def first_layers_and_route(model: Model, st: KVState, h_in: np.ndarray, k: Seque
         scores[i], kk, si = route(model, x, k[i])
         ks.append(kk)
         sel.append(si)
-    return RouteResult(H, scores, ks, sel, kv_new)
+        xs.append(x)
+    return RouteResult(H, scores, ks, sel, kv_new, np.stack(xs))
 
 
 def compaction(sel: Sequence[Sequence[int]], L: int, first: int = 1) -> List[List[int]]:
@@ -590,14 +592,15 @@ def prefill(model: Model, st: KVState, prompts: Sequence[np.ndarray], k: Sequenc
         for i in range(B):
             run_layer(l, i)
     scores = np.empty((B, sh.n_cand))
-    ks, sel = [], []
+    ks, sel, xs = [], [], []
     for i in range(B):
         K, V = st.get(c, i)
         x = router_input(sh, K, V, X[i][-1])
         scores[i], kk, si = route(model, x, k[i])
         ks.append(kk)
         sel.append(si)
-    rr = RouteResult(np.stack([X[i][-1] for i in range(B)]), scores, ks, sel, {})
+        xs.append(x)
+    rr = RouteResult(np.stack([X[i][-1] for i in range(B)]), scores, ks, sel, {}, np.stack(xs))
     if override_sel is not None:
         sel = override_sel(rr)
     rows = compaction(sel, L, sh.first_candidate)

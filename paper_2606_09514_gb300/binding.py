@@ -14,13 +14,15 @@ LIB_PATH = os.path.join(_HERE, "libbuddy.so")
 
 BUDDY_OK, BUDDY_ERR_ARG, BUDDY_ERR_RANGE, BUDDY_ERR_CUDA, BUDDY_ERR_DEVICE, BUDDY_ERR_STATE = range(6)
 BUDDY_DTYPE_F32, BUDDY_DTYPE_BF16 = 0, 1
+BUDDY_FEATURE = {"v": 0, "k": 1, "kv": 2}
+BUDDY_SKIP = {"zero": 0, "masked": 1}
 BUDDY_DEV_BAD_BUDGET, BUDDY_DEV_BAD_POSITION, BUDDY_DEV_BAD_SEQ, BUDDY_DEV_TIMEOUT = 1, 2, 4, 8
 
 EXPORTED = ["buddy_create", "buddy_destroy", "buddy_set_weights", "buddy_kv_append", "buddy_route",
             "buddy_decode_step", "buddy_decode_step_host", "buddy_set_options",
             "buddy_device_status", "buddy_budget_to_k", "buddy_error_string", "buddy_version",
             "buddy_set_profiling", "buddy_profile_read", "buddy_profile_class_name",
-            "buddy_route_noalloc"]
+            "buddy_route_noalloc", "buddy_set_budget_predictor", "buddy_get_paths"]
 PROF_CLASSES = ["check", "rmsnorm", "gemm_qkv", "qkv_finalize", "attention", "gemm_o", "gemm_gate_up",
                 "gemm_down", "route", "compact", "other", "gemm_fixup",
                 "attn_merge"]
@@ -33,6 +35,7 @@ class buddy_config(ctypes.Structure):
     _fields_ = [("n_layers", c_i32), ("d_model", c_i32), ("n_q_heads", c_i32), ("n_kv_heads", c_i32),
                 ("head_dim", c_i32), ("ffn_dim", c_i32), ("dm_hidden", c_i32), ("dtype", c_i32),
                 ("max_batch", c_i32), ("max_pos", c_i32), ("qkv_bias", c_i32),
+                ("feature", c_i32), ("ctx_layer", c_i32), ("skip_kv", c_i32), ("max_prefill_tokens", c_i32),
                 ("rms_eps", ctypes.c_float), ("rope_theta", ctypes.c_float)]
 
 
@@ -46,9 +49,13 @@ class buddy_dm_weights(ctypes.Structure):
                 ("omega", ctypes.c_float)]
 
 
+class buddy_predictor_weights(ctypes.Structure):
+    _fields_ = [("w1", c_p), ("b1", c_p), ("w2", c_p), ("b2", c_p), ("hidden", c_i32)]
+
+
 class buddy_kv_state(ctypes.Structure):
     _fields_ = [("k_cache", ctypes.POINTER(c_p)), ("v_cache", ctypes.POINTER(c_p)), ("seq_off", c_p),
-                ("cap", c_p), ("len", c_p), ("pool_sum", c_p), ("batch", c_i32)]
+                ("cap", c_p), ("len", c_p), ("pool_sum", c_p), ("batch", c_i32), ("layer_len", c_p)]
 
 
 class BuddyError(RuntimeError):
@@ -94,6 +101,10 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.buddy_route_noalloc.argtypes = [c_i32, c_i32, c_i32, c_i32, c_i32, c_i32, ctypes.POINTER(buddy_dm_weights),
                                         c_i32, c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p]
     lib.buddy_route_noalloc.restype = ctypes.c_int
+    lib.buddy_set_budget_predictor.argtypes = [c_p, ctypes.POINTER(buddy_predictor_weights)]
+    lib.buddy_set_budget_predictor.restype = ctypes.c_int
+    lib.buddy_get_paths.argtypes = [c_p, ctypes.POINTER(c_i32), c_i32]
+    lib.buddy_get_paths.restype = ctypes.c_int
     for name in ("buddy_create", "buddy_set_weights", "buddy_kv_append", "buddy_route", "buddy_decode_step",
                  "buddy_decode_step_host", "buddy_set_options", "buddy_device_status", "buddy_set_profiling",
                  "buddy_profile_read"):
@@ -140,7 +151,8 @@ class KVCache:
     """Per-layer K/V caches in the library's layout (head-major block of cap_i
     positions per sequence), positions len_i and the pooled first-layer sums."""
 
-    def __init__(self, n_layers: int, n_kv: int, head_dim: int, caps: Sequence[int], dtype, device):
+    def __init__(self, n_layers: int, n_kv: int, head_dim: int, caps: Sequence[int], dtype, device,
+                 masked: bool = False):
         caps = [int(c) for c in caps]
         self.batch = len(caps)
         self.n_kv, self.head_dim = n_kv, head_dim
@@ -156,12 +168,16 @@ class KVCache:
         self.cap = torch.tensor(caps, dtype=torch.int32, device=device)
         self.len = torch.zeros(self.batch, dtype=torch.int32, device=device)
         self.pool_sum = torch.zeros(self.batch, n_kv * head_dim, dtype=torch.float32, device=device)
+        # masked skip variant: positions each layer holds
+        self.layer_len = (torch.zeros(n_layers, self.batch, dtype=torch.int32, device=device) if masked
+                          else None)
         self._caps = caps
         self._off = off
         self._kp = (c_p * n_layers)(*[t.data_ptr() for t in self.k])
         self._vp = (c_p * n_layers)(*[t.data_ptr() for t in self.v])
         self.state = buddy_kv_state(self._kp, self._vp, self.seq_off.data_ptr(), self.cap.data_ptr(),
-                                    self.len.data_ptr(), self.pool_sum.data_ptr(), self.batch)
+                                    self.len.data_ptr(), self.pool_sum.data_ptr(), self.batch,
+                                    None if self.layer_len is None else self.layer_len.data_ptr())
 
     def view(self, which: str, layer: int, seq: int) -> torch.Tensor:
         """[n_kv, cap_i, hd] view of one sequence's block."""
@@ -187,11 +203,13 @@ class Context:
     """Owns a buddy_ctx handle; keeps the registered weight tensors alive."""
 
     def __init__(self, *, n_layers, d_model, n_q_heads, n_kv_heads, head_dim, ffn_dim, dm_hidden, dtype,
-                 max_batch, max_pos, qkv_bias, rms_eps, rope_theta):
+                 max_batch, max_pos, qkv_bias, rms_eps, rope_theta, feature="v", ctx_layer=0, skip_kv="zero",
+                 max_prefill_tokens=0):
         self.lib = load_library()
         cfg = buddy_config(n_layers, d_model, n_q_heads, n_kv_heads, head_dim, ffn_dim, dm_hidden,
                            BUDDY_DTYPE_BF16 if dtype == "bf16" else BUDDY_DTYPE_F32, max_batch, max_pos,
-                           1 if qkv_bias else 0, rms_eps, rope_theta)
+                           1 if qkv_bias else 0, BUDDY_FEATURE[feature], int(ctx_layer), BUDDY_SKIP[skip_kv],
+                           int(max_prefill_tokens), rms_eps, rope_theta)
         h = c_p()
         _check(self.lib.buddy_create(ctypes.byref(cfg), ctypes.byref(h)), "buddy_create")
         self.handle = h
@@ -199,11 +217,13 @@ class Context:
         self._keep: List = []
 
     @classmethod
-    def for_shape(cls, shape, max_batch: int, max_pos: int) -> "Context":
+    def for_shape(cls, shape, max_batch: int, max_pos: int, max_prefill_tokens: int = 0) -> "Context":
         return cls(n_layers=shape.n_layers, d_model=shape.d_model, n_q_heads=shape.n_q_heads,
                    n_kv_heads=shape.n_kv_heads, head_dim=shape.head_dim, ffn_dim=shape.ffn_dim,
                    dm_hidden=shape.dm_hidden, dtype=shape.dtype, max_batch=max_batch, max_pos=max_pos,
-                   qkv_bias=shape.qkv_bias, rms_eps=shape.rms_eps, rope_theta=shape.rope_theta)
+                   qkv_bias=shape.qkv_bias, rms_eps=shape.rms_eps, rope_theta=shape.rope_theta,
+                   feature=shape.feature, ctx_layer=shape.ctx_layer, skip_kv=shape.skip_kv,
+                   max_prefill_tokens=max_prefill_tokens)
 
     def close(self):
         if self.handle is not None and self.handle.value:
@@ -229,6 +249,25 @@ class Context:
                                dm["b2"].data_ptr(), None if prior is None else prior.data_ptr(), float(omega))
         _check(self.lib.buddy_set_weights(self.handle, arr, ctypes.byref(dmw)), "buddy_set_weights")
         self._keep = [layers, dm, prior]
+
+    def buddy_set_budget_predictor(self, pw: Optional[Dict[str, torch.Tensor]]):
+        """Registers the Budget Predictor ({"w1", "b1", "w2", "b2"}), or removes it (None)."""
+        if pw is None:
+            _check(self.lib.buddy_set_budget_predictor(self.handle, None), "buddy_set_budget_predictor")
+            return
+        bp = buddy_predictor_weights(pw["w1"].data_ptr(), pw["b1"].data_ptr(), pw["w2"].data_ptr(),
+                                     pw["b2"].data_ptr(), int(pw["w1"].shape[0]))
+        _check(self.lib.buddy_set_budget_predictor(self.handle, ctypes.byref(bp)), "buddy_set_budget_predictor")
+        self._pred = pw
+
+    def buddy_get_paths(self) -> Dict[str, str]:
+        """Which kernels this context runs (see include/buddy.h)."""
+        v = (c_i32 * 4)()
+        _check(self.lib.buddy_get_paths(self.handle, v, 4), "buddy_get_paths")
+        return {"gemm": "tcgen05 bf16 (TMA, TMEM)" if v[0] else "CUDA-core fp32",
+                "attention": "mma.sync tensor-core" if v[1] else "CUDA-core",
+                "rmsnorm": "inside the QKV and gate/up GEMMs" if v[2] else "separate kernel",
+                "split_k_fixup": "separate kernel" if v[3] else "last-arriving CTA"}
 
     def buddy_set_options(self, use_graph: bool):
         _check(self.lib.buddy_set_options(self.handle, 1 if use_graph else 0), "buddy_set_options")

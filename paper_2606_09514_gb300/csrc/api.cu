@@ -94,13 +94,19 @@ extern "C" int buddy_create(const buddy_config* cfg, buddy_ctx** out) {
       g.d_model != g.n_q_heads * g.head_dim || g.d_model % 64 != 0 || g.ffn_dim <= 0 ||
       g.ffn_dim % 8 != 0 || g.dm_hidden <= 0 || g.max_batch < 1 || g.max_batch > kMaxBatch ||
       g.max_pos < 1 || (g.dtype != BUDDY_DTYPE_F32 && g.dtype != BUDDY_DTYPE_BF16) ||
-      !(g.rms_eps > 0.f) || !(g.rope_theta > 0.f))
+      !(g.rms_eps > 0.f) || !(g.rope_theta > 0.f) ||
+      (g.feature != BUDDY_FEATURE_V && g.feature != BUDDY_FEATURE_K && g.feature != BUDDY_FEATURE_KV) ||
+      g.ctx_layer < 0 || g.ctx_layer > g.n_layers - 3 ||
+      (g.skip_kv != BUDDY_SKIP_ZERO && g.skip_kv != BUDDY_SKIP_MASKED) || g.max_prefill_tokens < 0 ||
+      g.max_prefill_tokens > 65536 || (g.dtype == BUDDY_DTYPE_BF16 && g.max_batch > 256))
     return BUDDY_ERR_ARG;
   buddy_ctx* x = new (std::nothrow) buddy_ctx();
   if (!x) return BUDDY_ERR_CUDA;
   Ctx& c = x->c;
   c.cfg = g;
-  c.L = g.n_layers; c.Lm = g.n_layers - 2; c.d = g.d_model; c.nq = g.n_q_heads;
+  c.L = g.n_layers; c.cl = g.ctx_layer; c.Lm = g.n_layers - 2 - g.ctx_layer; c.d = g.d_model; c.nq = g.n_q_heads;
+  c.feature = g.feature;
+  c.masked = g.skip_kv == BUDDY_SKIP_MASKED;
   c.nkv = g.n_kv_heads; c.hd = g.head_dim; c.F = g.ffn_dim; c.r = g.dm_hidden;
   c.qd = c.nq * c.hd; c.kvd = c.nkv * c.hd; c.qkvN = c.qd + 2 * c.kvd;
   c.maxB = g.max_batch; c.max_pos = g.max_pos; c.dtype = g.dtype;
@@ -139,6 +145,7 @@ extern "C" int buddy_create(const buddy_config* cfg, buddy_ctx** out) {
   if ((e = cudaMemset(c.status, 0, 4 * sizeof(int32_t))) != cudaSuccess ||
       (e = cudaMemset(c.attn_ctr, 0, B * c.nkv * sizeof(int32_t))) != cudaSuccess)
     return fail(e);
+  c.dm_u_cols = c.r;
   if ((e = cudaStreamCreateWithFlags(&x->cap_stream, cudaStreamNonBlocking)) != cudaSuccess) return fail(e);
   launch_rope_table(c.rope_cos, c.rope_sin, c.max_pos, c.hd, (double)g.rope_theta, x->cap_stream);
   if ((e = cudaGetLastError()) != cudaSuccess || (e = cudaStreamSynchronize(x->cap_stream)) != cudaSuccess)
@@ -179,6 +186,27 @@ extern "C" int buddy_set_weights(buddy_ctx* ctx, const buddy_layer_weights* laye
   return BUDDY_OK;
 }
 
+extern "C" int buddy_set_budget_predictor(buddy_ctx* ctx, const buddy_predictor_weights* bp) {
+  if (!ctx) return BUDDY_ERR_ARG;
+  Ctx& c = ctx->c;
+  if (bp && (!bp->w1 || !bp->b1 || !bp->w2 || !bp->b2 || bp->hidden < 1 || bp->hidden > 65536))
+    return BUDDY_ERR_ARG;
+  CK(cudaDeviceSynchronize());   // dm_u may be in use by queued work
+  for (auto& kv : c.graphs) cudaGraphExecDestroy(kv.second);
+  c.graphs.clear();
+  const int cols = c.r + (bp ? bp->hidden : 0);
+  if (cols > c.dm_u_cols) {
+    float* nu = nullptr;
+    CK(cudaMalloc(&nu, (size_t)c.maxB * cols * sizeof(float)));
+    cudaFree(c.dm_u);
+    c.dm_u = nu;
+    c.dm_u_cols = cols;
+  }
+  c.have_pred = bp != nullptr;
+  if (bp) c.pred = *bp;
+  return BUDDY_OK;
+}
+
 extern "C" int buddy_set_options(buddy_ctx* ctx, int32_t use_graph) {
   if (!ctx) return BUDDY_ERR_ARG;
   ctx->c.use_graph = use_graph ? 1 : 0;
@@ -188,6 +216,7 @@ extern "C" int buddy_set_options(buddy_ctx* ctx, int32_t use_graph) {
 static int check_kv(const Ctx& c, const buddy_kv_state* kv, int need_batch) {
   if (!kv || !kv->k_cache || !kv->v_cache || !kv->seq_off || !kv->cap || !kv->len || !kv->pool_sum)
     return BUDDY_ERR_ARG;
+  if (c.masked && !kv->layer_len) return BUDDY_ERR_ARG;
   if (kv->batch < need_batch || kv->batch < 1) return BUDDY_ERR_ARG;
   for (int l = 0; l < c.L; ++l)
     if (!kv->k_cache[l] || !kv->v_cache[l]) return BUDDY_ERR_ARG;
@@ -239,6 +268,16 @@ struct ProfScope {
     c.prof.push_back(rec);
   }
 };
+
+extern "C" int buddy_get_paths(buddy_ctx* ctx, int32_t* paths, int32_t n) {
+  if (!ctx || !paths || n < 0 || n > 4) return BUDDY_ERR_ARG;
+  const Ctx& c = ctx->c;
+  if (!c.have_weights) return BUDDY_ERR_STATE;
+  const int32_t v[4] = {c.use_tc ? 1 : 0, attention_tc(c) ? 1 : 0, (c.use_tc && c.tc_panel) ? 1 : 0,
+                        (c.use_tc && c.tc_defer) ? 1 : 0};
+  for (int i = 0; i < n; ++i) paths[i] = v[i];
+  return BUDDY_OK;
+}
 
 extern "C" int buddy_set_profiling(buddy_ctx* ctx, int32_t on) {
   if (!ctx) return BUDDY_ERR_ARG;
@@ -304,9 +343,9 @@ static void run_gemm(Ctx& c, int epi, GemmArgs a, int layer, int which, cudaStre
 static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, const float* src,
                           float* H, cudaStream_t s, bool prof) {
   const buddy_layer_weights& W = c.layers[l];
-  // The first layer feeds the router: its GEMM inputs are kept as bf16 hi + lo
-  // pairs so that its output is a continuous function of the inputs.
-  const bool split = c.split0 && l == 0;
+  // Layers 0..c feed the router: their GEMM inputs are kept as bf16 hi + lo
+  // pairs so that the routing input carries ~16 mantissa bits.
+  const bool split = c.split0 && l <= c.cl;
   const bool panel = c.use_tc && c.tc_panel;   // RMSNorms inside the QKV and gate/up GEMMs
   if (!panel) {
     ProfScope p(c, s, BUDDY_PROF_RMSNORM, 1, prof);
@@ -317,17 +356,20 @@ static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, c
   g.max_m = sel.n;
   g.split = split;
   g.W = W.w_qkv; g.X = c.xn; g.X_lo = c.xn_lo; g.N = c.qkvN; g.K = c.d; g.out_f32 = c.qkv;
-  float* pool = l == 0 ? kv.pool_sum : nullptr;
+  // the value-state feature is pooled in the QKV epilogue of the context
+  // layer; the other features by launch_pool_update
+  float* pool = (l == c.cl && c.feature == BUDDY_FEATURE_V) ? kv.pool_sum : nullptr;
   if (panel) {
     g.in_norm_src = src;
     g.in_norm_gamma = W.attn_norm;
     // no RMSNorm kernel in between: the first middle layer's QKV GEMM follows
     // the compaction kernel that writes its row count
-    g.count_late = l == 1;
+    g.count_late = l == c.cl + 1;
   }
   if (c.use_tc) {
     // bias, RoPE, q, cache append and pool update in the GEMM epilogue
     g.qkv_bias = W.b_qkv; g.kv_len = kv.len; g.kv_seq_off = kv.seq_off; g.kv_cap = kv.cap;
+    g.cache_len = cache_len(c, kv, l);
     g.kc = kv.k_cache[l]; g.vc = kv.v_cache[l]; g.q_out = c.q; g.pool = pool;
     run_gemm(c, EPI_QKV, g, l, 0, s, BUDDY_PROF_GEMM_QKV, prof);
   } else {
@@ -387,10 +429,14 @@ static int enqueue_step(buddy_ctx* x, const buddy_kv_state& kv, const StepIO& io
   const bool prof = c.profiling && !capture;
   {
     ProfScope p(c, s, BUDDY_PROF_CHECK, 1, prof);
-    launch_step_check(c, B, io.k, kv.len, kv.cap, 1, c.status, s);
+    launch_step_check(c, B, io.k, kv, 1, c.status, s);
   }
   const RowSel all{nullptr, nullptr, B};
-  enqueue_layer(c, kv, 0, all, io.h_in, io.h_out, s, prof);
+  for (int l = 0; l <= c.cl; ++l) enqueue_layer(c, kv, l, all, l == 0 ? io.h_in : io.h_out, io.h_out, s, prof);
+  if (c.feature != BUDDY_FEATURE_V) {
+    ProfScope p(c, s, BUDDY_PROF_ROUTE, 1, prof);
+    launch_pool_update(c, B, kv, s);
+  }
   {
     ProfScope p(c, s, BUDDY_PROF_ROUTE, 2, prof);
     launch_route(c, B, io.h_out, kv.pool_sum, kv.len, 1, io.k, c.mask, c.sel, c.scores, s);
@@ -410,14 +456,14 @@ static int enqueue_step(buddy_ctx* x, const buddy_kv_state& kv, const StepIO& io
   // read before any setup).  Graph conditional nodes would skip those launches
   // but cut the programmatic-dependent-launch overlap at every executed layer,
   // which costs more at the budgets of interest.
-  for (int l = 1; l < c.L - 1; ++l) {
+  for (int l = c.cl + 1; l < c.L - 1; ++l) {
     const RowSel sel{c.rows + (size_t)l * B, c.count + l, B};
     if (!prof || hcount[l] > 0) enqueue_layer(c, kv, l, sel, io.h_out, io.h_out, s, prof);
   }
   enqueue_layer(c, kv, c.L - 1, all, io.h_out, io.h_out, s, prof);
   {
     ProfScope p(c, s, BUDDY_PROF_OTHER, 1, prof);
-    launch_advance(c, B, kv.len, 1, nullptr, s);
+    launch_advance(c, B, kv.len, 1, nullptr, s, c.masked ? c.mask : nullptr, kv.layer_len, kv.batch);
   }
   if (io.mask_out) CK(cudaMemcpyAsync(io.mask_out, c.mask, (size_t)B * c.L, cudaMemcpyDeviceToDevice, s));
   if (io.rows_out)
@@ -443,6 +489,7 @@ static int run_step(buddy_ctx* x, const buddy_kv_state* kv, const StepIO& io, cu
   key.kvp.push_back(kv->cap);
   key.kvp.push_back(kv->len);
   key.kvp.push_back(kv->pool_sum);
+  key.kvp.push_back(kv->layer_len);
   auto it = c.graphs.find(key);
   if (it == c.graphs.end()) {
     if (c.graphs.size() >= 16) {   // bounded cache: drop an arbitrary old entry
@@ -516,7 +563,9 @@ extern "C" int buddy_route(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t bat
   if (!kv || !kv->len || !kv->pool_sum || !kv->cap || kv->batch < batch) return BUDDY_ERR_ARG;
   cudaStream_t s = (cudaStream_t)stream;
   // positions: the cache already holds the newest token (len >= 1)
-  launch_step_check(c, batch, k, kv->len, kv->cap, 0, c.status, s);
+  buddy_kv_state kvc = *kv;
+  kvc.layer_len = nullptr;   // only the context layer's pool and len are read
+  launch_step_check(c, batch, k, kvc, 0, c.status, s);
   launch_route(c, batch, h1, kv->pool_sum, kv->len, 0, k, mask_out, sel_out, scores_out, s);
   CK(cudaGetLastError());
   return BUDDY_OK;
@@ -534,9 +583,12 @@ extern "C" int buddy_kv_append(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t
   int rc = check_kv(c, kv, 1);
   if (rc) return rc;
   cudaStream_t s = (cudaStream_t)stream;
-  launch_kv_check(c, n_seq, seq_ids, n_new, kv->batch, kv->len, kv->cap, c.status, s);
+  int32_t* base = const_cast<int32_t*>(cache_len(c, *kv, layer));
+  launch_kv_check(c, n_seq, seq_ids, n_new, kv->batch, base, kv->cap, c.status, s);
   if (n_new > 0) launch_kv_append(c, *kv, layer, n_seq, seq_ids, n_new, k_new, v_new, s);
-  if (layer == 0) launch_pool_refresh(c, *kv, n_seq, seq_ids, n_new, s);
+  if (layer == c.cl) launch_pool_refresh(c, *kv, n_seq, seq_ids, n_new, s);
+  // the masked variant's per-layer length grows with its own appends
+  if (c.masked && n_new > 0) launch_advance(c, n_seq, base, n_new, seq_ids, s);
   if (advance && n_new > 0) launch_advance(c, n_seq, kv->len, n_new, seq_ids, s);
   CK(cudaGetLastError());
   return BUDDY_OK;

@@ -7,7 +7,7 @@
 //   * bf16 caches (G <= 8): the tensor-core loop of attn_tc.cuh (warp shares
 //     of the concatenated position streams, mma.sync contractions) and its
 //     span-merge kernel;
-//   * fp32 caches (and the opt-in per-layer persistent kernel): the CUDA-core
+//   * fp32 caches: the CUDA-core
 //     loop of attn_common.cuh.  Its work items are (row, KV head, span of P
 //     positions); P is derived on the device from the total number of
 //     positions so that there are about as many items as half the grid
@@ -59,7 +59,7 @@ static void attn_tc_impl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int
     occ_smem = smem;
   }
   const int grid = c.num_sms * std::max(1, std::min(occ, 4));
-  AttnArgs<bf16> A{q, sel.rows, sel.count, sel.n, c.nq, c.nkv, kv.len, kv.seq_off, kv.cap,
+  AttnArgs<bf16> A{q, sel.rows, sel.count, sel.n, c.nq, c.nkv, cache_len(c, kv, layer), kv.seq_off, kv.cap,
                    (const bf16*)kv.k_cache[layer], (const bf16*)kv.v_cache[layer], c.attn_max_chunks, c.attn_m,
                    c.attn_l, c.attn_acc, c.attn_ctr, (bf16*)out, (bf16*)out_lo, c.status, c.attn_meta};
   launch_k(attn_tc_kernel<HD, SPLIT>, grid, kTcaThreads, smem, s, c.pdl, A);
@@ -99,7 +99,7 @@ static void attn_impl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int la
     occ_smem = smem;
   }
   const int grid = c.num_sms * std::max(1, std::min(occ, 4));
-  AttnArgs<T> A{q, sel.rows, sel.count, sel.n, c.nq, c.nkv, kv.len, kv.seq_off, kv.cap,
+  AttnArgs<T> A{q, sel.rows, sel.count, sel.n, c.nq, c.nkv, cache_len(c, kv, layer), kv.seq_off, kv.cap,
                 (const T*)kv.k_cache[layer], (const T*)kv.v_cache[layer], c.attn_max_chunks, c.attn_m, c.attn_l,
                 c.attn_acc, c.attn_ctr, (T*)out, (T*)out_lo, c.status};
   launch_k(attn_kernel<T, HD, GP>, grid, kAttnThreads, smem, s, c.pdl, A);

@@ -73,7 +73,8 @@ struct TcParams {
   const float* bias;
   const float* rope_cos;
   const float* rope_sin;
-  const int32_t* len;
+  const int32_t* len;        // RoPE position of each sequence's token
+  const int32_t* cache_len;  // cache position of its new entry (len, or the layer's length)
   const int64_t* seq_off;
   const int32_t* cap;
   bf16* kc;
@@ -305,6 +306,7 @@ __device__ __forceinline__ void tc_apply4(const TcParams& p, int tile, int j, in
     const int head = n0 / hd, e0 = n0 - head * hd;
     const int seq = p.rows ? p.rows[j] : j;
     const int pos = p.len[seq];
+    const int cpos = p.cache_len[seq];
     float x[4], xp[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
@@ -328,7 +330,7 @@ __device__ __forceinline__ void tc_apply4(const TcParams& p, int tile, int j, in
           q[half + i] = hi[i];
         }
       } else {
-        bf16* k = p.kc + kv_offset(p.seq_off, p.cap, seq, p.nkv, hd, head - p.nq, pos) + e0;
+        bf16* k = p.kc + kv_offset(p.seq_off, p.cap, seq, p.nkv, hd, head - p.nq, cpos) + e0;
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           k[i] = from_f<bf16>(lo[i]);
@@ -337,7 +339,7 @@ __device__ __forceinline__ void tc_apply4(const TcParams& p, int tile, int j, in
       }
     } else {
       const int g = head - p.nq - p.nkv;
-      bf16* vv = p.vc + kv_offset(p.seq_off, p.cap, seq, p.nkv, hd, g, pos) + e0;
+      bf16* vv = p.vc + kv_offset(p.seq_off, p.cap, seq, p.nkv, hd, g, cpos) + e0;
       float* pl = p.pool ? p.pool + (size_t)seq * p.nkv * hd + g * hd + e0 : nullptr;
 #pragma unroll
       for (int i = 0; i < 4; ++i) {

@@ -519,6 +519,7 @@ static TcParams tc_params(const Ctx& c, const GemmArgs& a, size_t* smem_out) {
   p.rope_cos = c.rope_cos;
   p.rope_sin = c.rope_sin;
   p.len = a.kv_len;
+  p.cache_len = a.cache_len ? a.cache_len : a.kv_len;
   p.seq_off = a.kv_seq_off;
   p.cap = a.kv_cap;
   p.kc = (bf16*)a.kc;

@@ -49,7 +49,8 @@ struct GemmArgs {
   float* resid_dst;
   // EPI_QKV (tensor-core path): QKV finalisation fused into the epilogue
   const float* qkv_bias;
-  const int32_t* kv_len;
+  const int32_t* kv_len;       // RoPE positions (tokens of each sequence)
+  const int32_t* cache_len;    // where the layer's cache stores the new entry
   const int64_t* kv_seq_off;
   const int32_t* kv_cap;
   void* kc;
@@ -89,8 +90,8 @@ inline cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_
 
 // Kernel launchers (kernels.cu)
 void launch_rope_table(float* cos_t, float* sin_t, int max_pos, int hd, double theta, cudaStream_t s);
-void launch_step_check(const Ctx& c, int B, const int32_t* k, const int32_t* len, const int32_t* cap,
-                       int extra_pos, int32_t* status, cudaStream_t s);
+void launch_step_check(const Ctx& c, int B, const int32_t* k, const buddy_kv_state& kv, int extra_pos,
+                       int32_t* status, cudaStream_t s);
 void launch_kv_check(const Ctx& c, int n_seq, const int32_t* seq_ids, int n_new, int batch,
                      const int32_t* len, const int32_t* cap, int32_t* status, cudaStream_t s);
 void launch_rmsnorm(const Ctx& c, const float* H, RowSel sel, const float* gamma, void* xn, void* xn_lo,
@@ -108,7 +109,9 @@ void launch_route(const Ctx& c, int B, const float* h1, const float* pool, const
                   cudaStream_t s);
 void launch_compact(const Ctx& c, int B, const uint8_t* mask, const buddy_kv_state& kv,
                     int32_t* rows, int32_t* count, cudaStream_t s);
-void launch_advance(const Ctx& c, int B, int32_t* len, int by, const int32_t* seq_ids, cudaStream_t s);
+void launch_advance(const Ctx& c, int B, int32_t* len, int by, const int32_t* seq_ids, cudaStream_t s,
+                    const uint8_t* mask = nullptr, int32_t* layer_len = nullptr, int kv_batch = 0);
+void launch_pool_update(const Ctx& c, int B, const buddy_kv_state& kv, cudaStream_t s);
 void launch_kv_append(const Ctx& c, const buddy_kv_state& kv, int layer, int n_seq,
                       const int32_t* seq_ids, int n_new, const void* k_new, const void* v_new,
                       cudaStream_t s);
@@ -122,8 +125,11 @@ void launch_gemm_fix(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s); 
 
 struct Ctx {
   buddy_config cfg;
-  int L, Lm, d, nq, nkv, hd, F, r, qd, kvd, qkvN, maxB, max_pos;
+  // Lm = n_cand, the routed layers cl+1 .. L-2 (cl = the context layer)
+  int L, Lm, cl, d, nq, nkv, hd, F, r, qd, kvd, qkvN, maxB, max_pos;
   int dtype;
+  int feature = BUDDY_FEATURE_V;   // planner feature
+  bool masked = false;             // BUDDY_SKIP_MASKED: per-layer cache lengths
   size_t esz;
   int device, num_sms;
   bool pdl = true;             // programmatic dependent launch between step kernels
@@ -131,6 +137,9 @@ struct Ctx {
   bool have_weights = false;
   std::vector<buddy_layer_weights> layers;
   buddy_dm_weights dm{};
+  bool have_pred = false;          // Budget Predictor registered
+  buddy_predictor_weights pred{};
+  int dm_u_cols = 0;               // columns of dm_u: r + predictor hidden
 
   // scratch (device)
   float* rope_cos = nullptr;   // [max_pos, hd/2]
@@ -152,7 +161,7 @@ struct Ctx {
   float* attn_acc = nullptr;   // [maxB, nq, max_chunks, hd]
   int32_t* attn_ctr = nullptr; // [maxB, nkv] chunk arrivals (self-resetting)
   int32_t* attn_meta = nullptr;   // [maxB + 2] row prefix and share (tensor-core attention)
-  float* dm_u = nullptr;       // [maxB, r]
+  float* dm_u = nullptr;       // [maxB, r + predictor hidden]
   uint8_t* mask = nullptr;     // [maxB, L]
   int32_t* sel = nullptr;      // [maxB, Lm]
   float* scores = nullptr;     // [maxB, Lm]
@@ -199,5 +208,11 @@ struct Ctx {
   };
   std::map<GraphKey, cudaGraphExec_t> graphs;
 };
+
+// Positions layer l holds for each sequence (where its next entry goes):
+// layer_len[l] in the masked variant, else len.
+inline const int32_t* cache_len(const Ctx& c, const buddy_kv_state& kv, int l) {
+  return c.masked ? kv.layer_len + (size_t)l * kv.batch : kv.len;
+}
 
 }  // namespace buddy

@@ -30,8 +30,9 @@ void launch_rope_table(float* c, float* s, int max_pos, int hd, double theta, cu
 // Argument checks that need device data.  One CTA decides for the whole call
 // and publishes the abort flag that every later kernel of the call reads.
 // ---------------------------------------------------------------------------
-__global__ void step_check_kernel(int B, const int32_t* k, int Lm, const int32_t* len,
-                                  const int32_t* cap, int extra, int max_pos, int32_t* status) {
+__global__ void step_check_kernel(int B, const int32_t* k, int Lm, int k_min, const int32_t* len,
+                                  const int32_t* cap, int extra, int max_pos, const int32_t* layer_len,
+                                  int L, int kv_batch, int32_t* status) {
   pdl_wait();
   pdl_trigger();
   __shared__ int bad;
@@ -41,10 +42,15 @@ __global__ void step_check_kernel(int B, const int32_t* k, int Lm, const int32_t
   for (int i = threadIdx.x; i < B; i += blockDim.x) {
     if (k != nullptr) {
       const int ki = k[i];
-      if (ki < 1 || ki > Lm) b |= BUDDY_DEV_BAD_BUDGET;
+      if (ki < k_min || ki > Lm) b |= BUDDY_DEV_BAD_BUDGET;
     }
     const int n = len[i];
     if (n < 0 || n + extra > cap[i] || n + extra > max_pos) b |= BUDDY_DEV_BAD_POSITION;
+    if (layer_len != nullptr)
+      for (int l = 0; l < L; ++l) {
+        const int nl = layer_len[(size_t)l * kv_batch + i];
+        if (nl < 0 || nl > n) b |= BUDDY_DEV_BAD_POSITION;
+      }
   }
   if (b) atomicOr(&bad, b);
   __syncthreads();
@@ -54,13 +60,16 @@ __global__ void step_check_kernel(int B, const int32_t* k, int Lm, const int32_t
   }
 }
 
-void launch_step_check(const Ctx& c, int B, const int32_t* k, const int32_t* len, const int32_t* cap,
-                       int extra, int32_t* status, cudaStream_t s) {
-  launch_k(step_check_kernel, 1, 256, 0, s, c.pdl, B, k, c.Lm, len, cap, extra, c.max_pos, status);
+void launch_step_check(const Ctx& c, int B, const int32_t* k, const buddy_kv_state& kv, int extra,
+                       int32_t* status, cudaStream_t s) {
+  const int k_min = c.have_pred ? 0 : 1;   // 0 = "no budget": the Budget Predictor chooses
+  launch_k(step_check_kernel, 1, 256, 0, s, c.pdl, B, k, c.Lm, k_min, (const int32_t*)kv.len, kv.cap, extra,
+           c.max_pos, (const int32_t*)kv.layer_len, c.L, kv.batch, status);
 }
 
 __global__ void kv_check_kernel(int n_seq, const int32_t* ids, int n_new, int batch,
                                 const int32_t* len, const int32_t* cap, int max_pos, int32_t* status) {
+  // len: the positions the append starts at (len, or the layer's layer_len)
   pdl_wait();
   pdl_trigger();
   __shared__ int bad;
@@ -162,8 +171,8 @@ template <typename T>
 __global__ void __launch_bounds__(256) qkv_finalize_kernel(
     const float* __restrict__ qkv, const float* __restrict__ bias, const int32_t* rows,
     const int32_t* count, int n, int nq, int nkv, int hd, const float* __restrict__ rc,
-    const float* __restrict__ rs, const int32_t* len, const int64_t* seq_off, const int32_t* cap,
-    T* Kc, T* Vc, float* __restrict__ q_out, float* pool, const int32_t* status) {
+    const float* __restrict__ rs, const int32_t* len, const int32_t* cache_len, const int64_t* seq_off,
+    const int32_t* cap, T* Kc, T* Vc, float* __restrict__ q_out, float* pool, const int32_t* status) {
   pdl_wait();
   pdl_trigger();
   if (call_aborted(status)) return;
@@ -171,7 +180,8 @@ __global__ void __launch_bounds__(256) qkv_finalize_kernel(
   const int j = blockIdx.x;
   if (j >= m) return;
   const int i = rows ? rows[j] : j;
-  const int pos = len[i];
+  const int pos = len[i];          // RoPE position of the token
+  const int cpos = cache_len[i];   // where the layer's cache stores it
   const int half = hd / 2;
   const int N = (nq + 2 * nkv) * hd;
   const float* x = qkv + (size_t)j * N;
@@ -193,7 +203,7 @@ __global__ void __launch_bounds__(256) qkv_finalize_kernel(
       q_out[(size_t)j * nq * hd + c0 + half] = y2;
     } else {
       const int g = head - nq;
-      T* kp = Kc + kv_offset(seq_off, cap, i, nkv, hd, g, pos);
+      T* kp = Kc + kv_offset(seq_off, cap, i, nkv, hd, g, cpos);
       kp[e] = from_f<T>(y1);
       kp[e + half] = from_f<T>(y2);
     }
@@ -204,7 +214,7 @@ __global__ void __launch_bounds__(256) qkv_finalize_kernel(
     float v = x[vbase + t];
     if (bias) v += bias[vbase + t];
     const T vs = from_f<T>(v);
-    Vc[kv_offset(seq_off, cap, i, nkv, hd, g, pos) + e] = vs;
+    Vc[kv_offset(seq_off, cap, i, nkv, hd, g, cpos) + e] = vs;
     if (pool) pool[(size_t)i * nkv * hd + t] += to_f(vs);
   }
 }
@@ -212,37 +222,78 @@ __global__ void __launch_bounds__(256) qkv_finalize_kernel(
 void launch_qkv_finalize(const Ctx& c, const float* qkv, const float* bias, RowSel sel,
                          const buddy_kv_state& kv, int layer, float* q_out, float* pool,
                          cudaStream_t s) {
+  const int32_t* cl = cache_len(c, kv, layer);
   if (c.dtype == BUDDY_DTYPE_BF16)
     launch_k(qkv_finalize_kernel<bf16>, sel.n, 256, 0, s, c.pdl,
              qkv, bias, sel.rows, sel.count, sel.n, c.nq, c.nkv, c.hd, (const float*)c.rope_cos,
-             (const float*)c.rope_sin, (const int32_t*)kv.len, kv.seq_off, kv.cap, (bf16*)kv.k_cache[layer],
+             (const float*)c.rope_sin, (const int32_t*)kv.len, cl, kv.seq_off, kv.cap, (bf16*)kv.k_cache[layer],
              (bf16*)kv.v_cache[layer], q_out, pool, (const int32_t*)c.status);
   else
     launch_k(qkv_finalize_kernel<float>, sel.n, 256, 0, s, c.pdl,
              qkv, bias, sel.rows, sel.count, sel.n, c.nq, c.nkv, c.hd, (const float*)c.rope_cos,
-             (const float*)c.rope_sin, (const int32_t*)kv.len, kv.seq_off, kv.cap, (float*)kv.k_cache[layer],
+             (const float*)c.rope_sin, (const int32_t*)kv.len, cl, kv.seq_off, kv.cap, (float*)kv.k_cache[layer],
              (float*)kv.v_cache[layer], q_out, pool, (const int32_t*)c.status);
+}
+
+// ---------------------------------------------------------------------------
+// Pooled context update for the K and K + V planner features (Sec. 4.3,
+// Sec. 5.4): pool[i] += feature of the entry the context layer just stored at
+// position pos[i].  (The V feature is added in the QKV epilogue itself.)
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(256) pool_update_kernel(int B, int nkv, int hd, int feature,
+                                                          const int32_t* pos, const int64_t* seq_off,
+                                                          const int32_t* cap, const T* Kc, const T* Vc,
+                                                          float* pool, const int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
+  if (call_aborted(status)) return;
+  const int i = blockIdx.y;
+  const int x = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= B || x >= nkv * hd) return;
+  const int g = x / hd, e = x - g * hd;
+  const int64_t off = kv_offset(seq_off, cap, i, nkv, hd, g, pos[i]) + e;
+  float f = 0.f;
+  if (feature != BUDDY_FEATURE_V) f += to_f(Kc[off]);
+  if (feature != BUDDY_FEATURE_K) f += to_f(Vc[off]);
+  pool[(size_t)i * nkv * hd + x] += f;
+}
+
+void launch_pool_update(const Ctx& c, int B, const buddy_kv_state& kv, cudaStream_t s) {
+  const int l = c.cl;
+  dim3 g((c.kvd + 255) / 256, B);
+  if (c.dtype == BUDDY_DTYPE_BF16)
+    launch_k(pool_update_kernel<bf16>, g, 256, 0, s, c.pdl, B, c.nkv, c.hd, c.feature, cache_len(c, kv, l),
+             kv.seq_off, kv.cap, (const bf16*)kv.k_cache[l], (const bf16*)kv.v_cache[l], kv.pool_sum,
+             (const int32_t*)c.status);
+  else
+    launch_k(pool_update_kernel<float>, g, 256, 0, s, c.pdl, B, c.nkv, c.hd, c.feature, cache_len(c, kv, l),
+             kv.seq_off, kv.cap, (const float*)kv.k_cache[l], (const float*)kv.v_cache[l], kv.pool_sum,
+             (const int32_t*)c.status);
 }
 
 // ---------------------------------------------------------------------------
 // Router, part 1 (Sec. 4.3 + App. C.1 first linear layer):
 //   x_i = [ pool_sum[i] / (len[i] + len_bias), expanded over query heads ; h1[i] ]
-//   u[i][r] = SiLU(b1[r] + W1[r] . x_i)
-// One warp per hidden unit r and up to 8 sequences.
+//   u[i][unit] = SiLU(b1[unit] + W1[unit] . x_i)
+// for the Decision Module's r hidden units and, after them, the Budget
+// Predictor's rp hidden units (same input, Sec. 4.4).  One warp per hidden
+// unit and up to 8 sequences; u has r + rp columns.
 // ---------------------------------------------------------------------------
 constexpr int kRouteRows = 8;
 
 __global__ void __launch_bounds__(256) route_hidden_kernel(
     int B, int d, int hd, int group, int nkv, const float* __restrict__ h1,
     const float* __restrict__ pool, const int32_t* len, int len_bias, const float* __restrict__ w1,
-    const float* __restrict__ b1, int r, float* __restrict__ u, const int32_t* status) {
+    const float* __restrict__ b1, int r, const float* __restrict__ pw1, const float* __restrict__ pb1, int rp,
+    float* __restrict__ u, const int32_t* status) {
   pdl_wait();
   pdl_trigger();
   if (call_aborted(status)) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int unit = blockIdx.x * 8 + warp;
   const int i0 = blockIdx.y * kRouteRows;
-  if (unit >= r) return;
+  if (unit >= r + rp) return;
   const int nr = min(kRouteRows, B - i0);
   float inv[kRouteRows];
 #pragma unroll
@@ -250,7 +301,7 @@ __global__ void __launch_bounds__(256) route_hidden_kernel(
   float acc[kRouteRows];
 #pragma unroll
   for (int t = 0; t < kRouteRows; ++t) acc[t] = 0.f;
-  const float* wr = w1 + (size_t)unit * 2 * d;
+  const float* wr = unit < r ? w1 + (size_t)unit * 2 * d : pw1 + (size_t)(unit - r) * 2 * d;
   const int kvd = nkv * hd;
   // pooled part: x[k] = pool[(k / hd) / group * hd + k % hd] / n
   for (int k = lane * 4; k < d; k += 128) {
@@ -282,35 +333,63 @@ __global__ void __launch_bounds__(256) route_hidden_kernel(
 #pragma unroll
     for (int t = 0; t < kRouteRows; ++t)
       if (t == lane) v = acc[t];
-    u[(size_t)(i0 + lane) * r + unit] = silu_f(v + b1[unit]);
+    u[(size_t)(i0 + lane) * (r + rp) + unit] = silu_f(v + (unit < r ? b1[unit] : pb1[unit - r]));
   }
 }
 
-// Router, part 2: s' = W2 u + b2 + omega p~, then the deterministic top-k
-// (Eq. 2): layer l is selected iff fewer than k_i layers rank above it, where
-// l' ranks above l when s'[l'] > s'[l], or s'[l'] == s'[l] and l' < l.
-// One CTA per sequence.
-__global__ void __launch_bounds__(64) route_select_kernel(
-    int Lm, int r, const float* __restrict__ u, const float* __restrict__ w2,
-    const float* __restrict__ b2, const float* __restrict__ prior, float omega, const int32_t* k,
+// Router, part 2: s' = W2 u + b2 + omega p~ over the Lm routed layers
+// first .. first + Lm - 1, then the deterministic top-k (Eq. 2): layer l is
+// selected iff fewer than k_i layers rank above it, where l' ranks above l
+// when s'[l'] > s'[l], or s'[l'] == s'[l] and l' < l.  A budget k_i = 0 takes
+// the Budget Predictor's k^ = 1 + argmax of its logits (ties to the smaller
+// k, Sec. 4.4).  Layers below `first` and the last layer are always set in
+// the mask.  One CTA per sequence; warps score layers (lanes split the dot
+// product).
+__global__ void __launch_bounds__(128) route_select_kernel(
+    int Lm, int first, int r, int rp, const float* __restrict__ u, const float* __restrict__ w2,
+    const float* __restrict__ b2, const float* __restrict__ prior, float omega,
+    const float* __restrict__ pw2, const float* __restrict__ pb2, const int32_t* k,
     uint8_t* mask, int32_t* sel, float* scores, const int32_t* status) {
   pdl_wait();
   pdl_trigger();
   if (call_aborted(status)) return;
   const int i = blockIdx.x;
-  extern __shared__ float s[];           // [Lm]
+  extern __shared__ float s[];           // [Lm] scores, then [Lm] predictor logits
   __shared__ int flag[kMaxLayers];
-  const float* ui = u + (size_t)i * r;
-  for (int l = threadIdx.x; l < Lm; l += blockDim.x) {
+  __shared__ int kpred;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  const float* ui = u + (size_t)i * (r + rp);
+  const int ki0 = k[i];
+  const bool predict = ki0 == 0 && pw2 != nullptr;
+  for (int l = warp; l < (predict ? 2 * Lm : Lm); l += nw) {
+    const bool pl = l >= Lm;
+    const int row = pl ? l - Lm : l;
+    const float* w = pl ? pw2 + (size_t)row * rp : w2 + (size_t)row * r;
+    const float* x = pl ? ui + r : ui;
+    const int n = pl ? rp : r;
     float a = 0.f;
-    const float* w = w2 + (size_t)l * r;
-    for (int t = 0; t < r; ++t) a += w[t] * ui[t];
-    a += b2[l];
-    if (prior) a += omega * prior[l];
-    s[l] = a;
+    for (int t = lane; t < n; t += 32) a += w[t] * x[t];
+    a = warp_sum(a);
+    if (lane == 0) {
+      if (pl) {
+        s[l] = a + pb2[row];
+      } else {
+        a += b2[row];
+        if (prior) a += omega * prior[row];
+        s[l] = a;
+      }
+    }
   }
   __syncthreads();
-  const int ki = k[i];
+  if (threadIdx.x == 0) {
+    int best = 0;
+    if (predict)
+      for (int t = 1; t < Lm; ++t)
+        if (s[Lm + t] > s[Lm + best]) best = t;
+    kpred = predict ? best + 1 : ki0;
+  }
+  __syncthreads();
+  const int ki = kpred;
   for (int l = threadIdx.x; l < Lm; l += blockDim.x) {
     int rank = 0;
     const float v = s[l];
@@ -318,31 +397,33 @@ __global__ void __launch_bounds__(64) route_select_kernel(
     flag[l] = rank < ki;
   }
   __syncthreads();
-  const int L = Lm + 2;
+  const int L = Lm + first + 1;
   for (int l = threadIdx.x; l < Lm; l += blockDim.x) {
     if (scores) scores[(size_t)i * Lm + l] = s[l];
-    if (mask) mask[(size_t)i * L + l + 1] = (uint8_t)flag[l];
+    if (mask) mask[(size_t)i * L + first + l] = (uint8_t)flag[l];
     if (sel) {
       int before = 0;
       for (int t = 0; t < l; ++t) before += flag[t];
-      if (flag[l]) sel[(size_t)i * Lm + before] = l + 1;
+      if (flag[l]) sel[(size_t)i * Lm + before] = first + l;
       if (l >= ki) sel[(size_t)i * Lm + l] = -1;
     }
   }
-  if (threadIdx.x == 0 && mask) {
-    mask[(size_t)i * L] = 1;
-    mask[(size_t)i * L + L - 1] = 1;
-  }
+  if (mask)
+    for (int l = threadIdx.x; l < first; l += blockDim.x) mask[(size_t)i * L + l] = 1;
+  if (threadIdx.x == 0 && mask) mask[(size_t)i * L + L - 1] = 1;
 }
 
 void launch_route(const Ctx& c, int B, const float* h1, const float* pool, const int32_t* len,
                   int len_bias, const int32_t* k, uint8_t* mask, int32_t* sel, float* scores,
                   cudaStream_t s) {
-  dim3 g1((c.r + 7) / 8, (B + kRouteRows - 1) / kRouteRows);
+  const int rp = c.have_pred ? c.pred.hidden : 0;
+  dim3 g1((c.r + rp + 7) / 8, (B + kRouteRows - 1) / kRouteRows);
   launch_k(route_hidden_kernel, g1, 256, 0, s, c.pdl, B, c.d, c.hd, c.nq / c.nkv, c.nkv, h1, pool, len,
-           len_bias, c.dm.w1, c.dm.b1, c.r, c.dm_u, (const int32_t*)c.status);
-  launch_k(route_select_kernel, B, 64, c.Lm * sizeof(float), s, c.pdl, c.Lm, c.r, (const float*)c.dm_u,
-           c.dm.w2, c.dm.b2, c.dm.prior, c.dm.omega, k, mask, sel, scores, (const int32_t*)c.status);
+           len_bias, c.dm.w1, c.dm.b1, c.r, c.have_pred ? c.pred.w1 : nullptr, c.have_pred ? c.pred.b1 : nullptr,
+           rp, c.dm_u, (const int32_t*)c.status);
+  launch_k(route_select_kernel, B, 128, 2 * c.Lm * sizeof(float), s, c.pdl, c.Lm, c.cl + 1, c.r, rp,
+           (const float*)c.dm_u, c.dm.w2, c.dm.b2, c.dm.prior, c.dm.omega, c.have_pred ? c.pred.w2 : nullptr,
+           c.have_pred ? c.pred.b2 : nullptr, k, mask, sel, scores, (const int32_t*)c.status);
 }
 
 // ---------------------------------------------------------------------------
@@ -356,7 +437,7 @@ __global__ void __launch_bounds__(1024) compact_kernel(int B, int L, int nkv, in
                                                        const uint8_t* __restrict__ mask,
                                                        LayerPtrs ptrs, const int32_t* len,
                                                        const int64_t* seq_off, const int32_t* cap,
-                                                       int32_t* rows, int32_t* count,
+                                                       int32_t* rows, int32_t* count, int zero_fill,
                                                        const int32_t* status) {
   pdl_wait();
   pdl_trigger();
@@ -387,8 +468,9 @@ __global__ void __launch_bounds__(1024) compact_kernel(int B, int L, int nkv, in
     __syncthreads();
   }
   if (threadIdx.x == 0) count[l] = carry;
-  // zero K/V at the new position for sequences that skip this layer
-  if (l == 0 || l == L - 1) return;
+  // zero K/V at the new position for sequences that skip this layer (the
+  // masked variant stores nothing)
+  if (!zero_fill || l == 0 || l == L - 1) return;
   T* Kc = (T*)ptrs.k[l];
   T* Vc = (T*)ptrs.v[l];
   const int kvd = nkv * hd;
@@ -413,17 +495,18 @@ void launch_compact(const Ctx& c, int B, const uint8_t* mask, const buddy_kv_sta
   }
   if (c.dtype == BUDDY_DTYPE_BF16)
     launch_k(compact_kernel<bf16>, c.L, 1024, 0, s, c.pdl, B, c.L, c.nkv, c.hd, mask, p,
-             (const int32_t*)kv.len, kv.seq_off, kv.cap, rows, count, (const int32_t*)c.status);
+             (const int32_t*)kv.len, kv.seq_off, kv.cap, rows, count, c.masked ? 0 : 1, (const int32_t*)c.status);
   else
     launch_k(compact_kernel<float>, c.L, 1024, 0, s, c.pdl, B, c.L, c.nkv, c.hd, mask, p,
-             (const int32_t*)kv.len, kv.seq_off, kv.cap, rows, count, (const int32_t*)c.status);
+             (const int32_t*)kv.len, kv.seq_off, kv.cap, rows, count, c.masked ? 0 : 1, (const int32_t*)c.status);
 }
 
 // ---------------------------------------------------------------------------
-// Position advance: len[i] += by  (for i < B, or for the listed sequences).
+// Position advance: len[i] += by  (for i < B, or for the listed sequences);
+// with a mask (decode step, masked variant) also layer_len[l][i] += mask[i][l].
 // ---------------------------------------------------------------------------
-__global__ void advance_kernel(int B, int32_t* len, int by, const int32_t* ids,
-                               const int32_t* status) {
+__global__ void advance_kernel(int B, int32_t* len, int by, const int32_t* ids, const uint8_t* mask, int L,
+                               int32_t* layer_len, int kv_batch, const int32_t* status) {
   pdl_wait();
   pdl_trigger();
   if (call_aborted(status)) return;
@@ -431,10 +514,14 @@ __global__ void advance_kernel(int B, int32_t* len, int by, const int32_t* ids,
   if (t >= B) return;
   const int i = ids ? ids[t] : t;
   len[i] += by;
+  if (mask != nullptr)
+    for (int l = 0; l < L; ++l) layer_len[(size_t)l * kv_batch + i] += mask[(size_t)t * L + l];
 }
 
-void launch_advance(const Ctx& c, int B, int32_t* len, int by, const int32_t* ids, cudaStream_t s) {
-  launch_k(advance_kernel, (B + 255) / 256, 256, 0, s, c.pdl, B, len, by, ids, (const int32_t*)c.status);
+void launch_advance(const Ctx& c, int B, int32_t* len, int by, const int32_t* ids, cudaStream_t s,
+                    const uint8_t* mask, int32_t* layer_len, int kv_batch) {
+  launch_k(advance_kernel, (B + 255) / 256, 256, 0, s, c.pdl, B, len, by, ids, mask, c.L, layer_len, kv_batch,
+           (const int32_t*)c.status);
 }
 
 // ---------------------------------------------------------------------------
@@ -465,10 +552,10 @@ __global__ void __launch_bounds__(256) kv_append_kernel(int n_new, int nkv, int 
 }
 
 template <typename T>
-__global__ void __launch_bounds__(256) pool_refresh_kernel(int n_new, int nkv, int hd,
+__global__ void __launch_bounds__(256) pool_refresh_kernel(int n_new, int nkv, int hd, int feature,
                                                            const int32_t* ids, const int32_t* len,
                                                            const int64_t* seq_off,
-                                                           const int32_t* cap, const T* V0,
+                                                           const int32_t* cap, const T* K0, const T* V0,
                                                            float* pool, const int32_t* status) {
   pdl_wait();
   pdl_trigger();
@@ -479,22 +566,28 @@ __global__ void __launch_bounds__(256) pool_refresh_kernel(int n_new, int nkv, i
   if (x >= kvd) return;
   const int g = x / hd, e = x - g * hd;
   const int n = len[s] + n_new;
-  const T* base = V0 + kv_offset(seq_off, cap, s, nkv, hd, g, 0) + e;
+  const int64_t off = kv_offset(seq_off, cap, s, nkv, hd, g, 0) + e;
   float acc = 0.f;
-  for (int p = 0; p < n; ++p) acc += to_f(base[(size_t)p * hd]);
+  for (int p = 0; p < n; ++p) {
+    float f = 0.f;
+    if (feature != BUDDY_FEATURE_V) f += to_f(K0[off + (size_t)p * hd]);
+    if (feature != BUDDY_FEATURE_K) f += to_f(V0[off + (size_t)p * hd]);
+    acc += f;
+  }
   pool[(size_t)s * kvd + x] = acc;
 }
 
 void launch_kv_append(const Ctx& c, const buddy_kv_state& kv, int layer, int n_seq,
                       const int32_t* ids, int n_new, const void* kn, const void* vn, cudaStream_t s) {
   dim3 g(n_new, n_seq);
+  const int32_t* base = cache_len(c, kv, layer);
   if (c.dtype == BUDDY_DTYPE_BF16)
-    kv_append_kernel<bf16><<<g, 256, 0, s>>>(n_new, c.nkv, c.hd, ids, kv.len, kv.seq_off, kv.cap,
+    kv_append_kernel<bf16><<<g, 256, 0, s>>>(n_new, c.nkv, c.hd, ids, base, kv.seq_off, kv.cap,
                                              (const bf16*)kn, (const bf16*)vn,
                                              (bf16*)kv.k_cache[layer], (bf16*)kv.v_cache[layer],
                                              c.status);
   else
-    kv_append_kernel<float><<<g, 256, 0, s>>>(n_new, c.nkv, c.hd, ids, kv.len, kv.seq_off, kv.cap,
+    kv_append_kernel<float><<<g, 256, 0, s>>>(n_new, c.nkv, c.hd, ids, base, kv.seq_off, kv.cap,
                                               (const float*)kn, (const float*)vn,
                                               (float*)kv.k_cache[layer], (float*)kv.v_cache[layer],
                                               c.status);
@@ -503,13 +596,16 @@ void launch_kv_append(const Ctx& c, const buddy_kv_state& kv, int layer, int n_s
 void launch_pool_refresh(const Ctx& c, const buddy_kv_state& kv, int n_seq, const int32_t* ids,
                          int n_new, cudaStream_t s) {
   dim3 g((c.kvd + 255) / 256, n_seq);
+  const int l = c.cl;
+  const int32_t* base = cache_len(c, kv, l);
   if (c.dtype == BUDDY_DTYPE_BF16)
-    pool_refresh_kernel<bf16><<<g, 256, 0, s>>>(n_new, c.nkv, c.hd, ids, kv.len, kv.seq_off, kv.cap,
-                                                (const bf16*)kv.v_cache[0], kv.pool_sum, c.status);
+    pool_refresh_kernel<bf16><<<g, 256, 0, s>>>(n_new, c.nkv, c.hd, c.feature, ids, base, kv.seq_off, kv.cap,
+                                                (const bf16*)kv.k_cache[l], (const bf16*)kv.v_cache[l],
+                                                kv.pool_sum, c.status);
   else
-    pool_refresh_kernel<float><<<g, 256, 0, s>>>(n_new, c.nkv, c.hd, ids, kv.len, kv.seq_off,
-                                                 kv.cap, (const float*)kv.v_cache[0], kv.pool_sum,
-                                                 c.status);
+    pool_refresh_kernel<float><<<g, 256, 0, s>>>(n_new, c.nkv, c.hd, c.feature, ids, base, kv.seq_off,
+                                                 kv.cap, (const float*)kv.k_cache[l],
+                                                 (const float*)kv.v_cache[l], kv.pool_sum, c.status);
 }
 
 }  // namespace buddy

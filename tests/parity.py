@@ -53,6 +53,28 @@ def adopt_routes(o_scores: np.ndarray, o_sel: Sequence[Sequence[int]], g_sel: Se
     return out, fails, adopted
 
 
+def adopt_budgets(o_k: Sequence[int], g_k: Sequence[int], logits: Sequence[np.ndarray],
+                  given: Sequence[int]) -> Tuple[List[int], List[str]]:
+    """Budgets the oracle continues with.  Where the Budget Predictor chose
+    (given[i] == 0) and the GPU's k^ differs from the oracle's, the oracle
+    adopts it if both are within ROUTE_MARGIN of the largest oracle logit (a
+    near-tie of the argmax, the same rule as for the layer ranking)."""
+    out, fails = [], []
+    for i, (ok, gk) in enumerate(zip(o_k, g_k)):
+        if ok == gk:
+            out.append(ok)
+            continue
+        if int(given[i]) == 0 and logits[i] is not None:
+            lg = np.asarray(logits[i], dtype=np.float64)
+            top = lg.max()
+            if 1 <= gk <= len(lg) and top - lg[gk - 1] < ROUTE_MARGIN and top - lg[ok - 1] < ROUTE_MARGIN:
+                out.append(gk)
+                continue
+        fails.append(f"seq {i}: gpu budget {gk} vs oracle {ok} (given {given[i]})")
+        out.append(ok)
+    return out, fails
+
+
 def max_rel_err(g: np.ndarray, o: np.ndarray) -> float:
     g = np.asarray(g, dtype=np.float64)
     o = np.asarray(o, dtype=np.float64)

@@ -56,7 +56,9 @@ def test_invalid_configs_rejected_before_any_cuda_call(lib):
                 dtype=0, max_batch=4, max_pos=64, qkv_bias=0, rms_eps=1e-5, rope_theta=1e4)
     bad_cases = [dict(n_layers=2), dict(head_dim=96), dict(n_kv_heads=3), dict(d_model=320),
                  dict(ffn_dim=700), dict(ffn_dim=0), dict(max_batch=0), dict(max_batch=5000), dict(max_pos=0),
-                 dict(dtype=7), dict(rms_eps=0.0), dict(n_q_heads=36, n_kv_heads=4, d_model=36 * 64)]
+                 dict(dtype=7), dict(rms_eps=0.0), dict(n_q_heads=36, n_kv_heads=4, d_model=36 * 64),
+                 dict(feature=3), dict(feature=-1), dict(ctx_layer=6), dict(ctx_layer=-1), dict(skip_kv=2),
+                 dict(max_prefill_tokens=-1), dict(max_prefill_tokens=70000), dict(dtype=1, max_batch=257)]
     for bad in bad_cases:
         cfg = B.buddy_config(**{**good, **bad})
         assert lib.buddy_create(ctypes.byref(cfg), ctypes.byref(h)) == B.BUDDY_ERR_ARG, bad
@@ -64,6 +66,7 @@ def test_invalid_configs_rejected_before_any_cuda_call(lib):
     assert lib.buddy_decode_step(None, None, 1, None, None, None, None, None, None, None, None) == B.BUDDY_ERR_ARG
     assert lib.buddy_route(None, None, 1, None, None, None, None, None, None) == B.BUDDY_ERR_ARG
     assert lib.buddy_kv_append(None, None, 0, 1, None, 1, None, None, 0, None) == B.BUDDY_ERR_ARG
+    assert lib.buddy_set_budget_predictor(None, None) == B.BUDDY_ERR_ARG
     assert lib.buddy_error_string(B.BUDDY_ERR_RANGE) == b"value out of range"
     assert lib.buddy_version() >= 1
 
@@ -73,7 +76,8 @@ def test_ctypes_structs_match_c_layout():
     binding's ctypes layouts."""
     from paper_2606_09514_gb300 import binding as B
     structs = {"buddy_config": B.buddy_config, "buddy_layer_weights": B.buddy_layer_weights,
-               "buddy_dm_weights": B.buddy_dm_weights, "buddy_kv_state": B.buddy_kv_state}
+               "buddy_dm_weights": B.buddy_dm_weights, "buddy_kv_state": B.buddy_kv_state,
+               "buddy_predictor_weights": B.buddy_predictor_weights}
     lines = ['#include <stdio.h>', '#include <stddef.h>', f'#include "{HEADER}"', 'int main(void){']
     for n, cls in structs.items():
         lines.append(f'printf("{n} %zu\\n", sizeof({n}));')

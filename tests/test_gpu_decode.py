@@ -25,16 +25,34 @@ def _oracle_for(dw, gen_device="cuda"):
     model = A.build_model(s, w.seed, layer_source=lambda l: synth.layer_weights(s, w.seed, l, gen_device),
                           dm_source=lambda: synth.dm_weights(s, w.seed, gen_device),
                           prior=dw.prior, omega=0.1 if dw.prior is not None else 0.0,
-                          cache_layers=s.n_layers)
+                          cache_layers=s.n_layers,
+                          predictor_source=lambda: synth.predictor_weights(s, w.seed, gen_device))
     st = A.build_state(s, w.seed, w.contexts(), gen_device=gen_device)
     return model, st
+
+
+def adopt(model, rr, g_mask, k_given):
+    """Near-tie rules: the oracle takes the GPU's budget where the Budget
+    Predictor's argmax is a near-tie, then the GPU's set where the layer
+    ranking is.  Returns (sets, budgets, failures, adopted)."""
+    first = model.shape.first_candidate
+    g_sel = P.sel_from_mask(g_mask, first)
+    g_k = [len(x) for x in g_sel]
+    logits = [O.predictor_logits(model.predictor, rr.x[i]) if model.predictor is not None else None
+              for i in range(len(g_sel))]
+    ks, fails_k = P.adopt_budgets(rr.k, g_k, logits, k_given)
+    o_sel = [rr.sel[i] if ks[i] == rr.k[i] else O.top_k_layers(rr.scores[i], ks[i], first)
+             for i in range(len(ks))]
+    sel, fails, n = P.adopt_routes(rr.scores, o_sel, g_sel, ks, first)
+    return sel, ks, fails_k + fails, n
 
 
 def run_parity(w, steps=None, use_graph=False, prior=False, check_kv=True):
     dw = D.build(w, use_graph=use_graph, prior=prior)
     model, st = _oracle_for(dw)
     s = w.shape
-    B, L, Lm = w.batch, s.n_layers, s.l_mid
+    B, L, Lm = w.batch, s.n_layers, s.n_cand
+    masked = s.skip_kv == "masked"
     dev = "cuda"
     h_out = torch.empty(B, s.d_model, device=dev)
     mask = torch.empty(B, L, dtype=torch.uint8, device=dev)
@@ -47,26 +65,26 @@ def run_parity(w, steps=None, use_graph=False, prior=False, check_kv=True):
     adopted_total = 0
     for t in range(steps or w.steps):
         n_before = list(st.n)
+        ll_before = dw.kv.layer_len.cpu().numpy().copy() if masked else None
         h_in = synth.workload_h_in(w, t, dev)
         dw.ctx.buddy_decode_step(dw.kv, h_in, dw.k, h_out, mask, rows, count, scores)
         torch.cuda.synchronize()
         assert dw.ctx.buddy_device_status() == 0
         g_mask = mask.cpu().numpy()
-        g_sel = P.sel_from_mask(g_mask)
         info = {}
 
-        def override(route):
-            sel, fails, n = P.adopt_routes(route.scores, route.sel, g_sel, k)
-            info["fails"], info["n"] = fails, n
+        def override(rr):
+            sel, ks, fails, n = adopt(model, rr, g_mask, k)
+            info["fails"], info["n"], info["k"] = fails, n, ks
             return sel
 
         res = O.decode_step(model, st, A.to_f64(h_in), k, override_sel=override)
         assert not info["fails"], info["fails"]
         adopted_total += info["n"]
         # scores agree well inside the near-tie margin
-        np.testing.assert_allclose(scores.cpu().numpy(), res.scores, rtol=0, atol=P.ROUTE_MARGIN / 4)
-        # exactly k middle layers + first + last
-        np.testing.assert_array_equal(g_mask.sum(1), k + 2)
+        np.testing.assert_allclose(scores.cpu().numpy(), res.scores, rtol=0, atol=P.ROUTE_MARGIN / 2)
+        # exactly k routed layers + the always-executed ones
+        np.testing.assert_array_equal(g_mask.sum(1), np.asarray(info["k"]) + s.ctx_layer + 2)
         # compaction: bit-exact
         g_count = count.cpu().numpy()
         g_rows = rows.cpu().numpy()
@@ -80,19 +98,26 @@ def run_parity(w, steps=None, use_graph=False, prior=False, check_kv=True):
             worst = max(worst, e)
             assert e < tol, (t, i, e)
         # KV written this step: real entries match, skipped layers hold zeros
+        # (zero variant) or nothing (masked variant: the layer's length grows
+        # only where it executed)
         if check_kv:
             for l in range(L):
                 for i in range(B):
-                    pos = n_before[i]
+                    pos = int(ll_before[l, i]) if masked else n_before[i]
                     gk = dw.kv.view("k", l, i)[:, pos, :].float().cpu().numpy()
                     gv = dw.kv.view("v", l, i)[:, pos, :].float().cpu().numpy()
-                    ok, ov = res.kv_new[(l, i)]
                     if g_mask[i, l]:
+                        ok, ov = res.kv_new[(l, i)]
                         assert P.max_rel_err(gk, ok) < P.KV_TOL[s.dtype] and P.max_rel_err(gv, ov) < P.KV_TOL[s.dtype]
-                    else:
+                    elif not masked:
                         assert not gk.any() and not gv.any()
+            if masked:
+                np.testing.assert_array_equal(dw.kv.layer_len.cpu().numpy(), ll_before + g_mask.T)
     # positions advanced by one per step
     np.testing.assert_array_equal(dw.kv.len.cpu().numpy(), np.asarray(st.n))
+    if masked:
+        for l in range(L):
+            np.testing.assert_array_equal(dw.kv.layer_len[l].cpu().numpy(), [st.length(l, i) for i in range(B)])
     return worst, adopted_total
 
 
@@ -128,6 +153,19 @@ def test_decode_parity_three_rows_graph_prior():
     w = C.scaled(C.T_QWEN, ctx=[0, 129, 700], k=[1, 5, 3], name="t-qwen-b3")
     worst, _ = run_parity(w, steps=3, use_graph=True, prior=True)
     assert worst < 2e-2
+
+
+@pytest.mark.parametrize("w", C.T_VARIANTS, ids=lambda w: w.name)
+def test_decode_parity_router_variants(w):
+    """K and K+V planner features, a context layer c > 0 with the Budget
+    Predictor choosing some budgets, and the masked skip-KV variant."""
+    worst, _ = run_parity(w)
+    assert worst < P.HIDDEN_TOL[w.shape.dtype]
+
+
+def test_router_variants_graph_prior():
+    run_parity(C.T_VARIANTS[1], steps=2, use_graph=True, prior=True)
+    run_parity(C.T_VARIANTS[2], steps=2, use_graph=True, prior=True)
 
 
 def test_graph_replay_equals_direct_launches():

@@ -82,9 +82,13 @@ def test_fullsize_trajectory_parity(w, sampled):
                     gpu_masks=[r["mask"] for r in rec])
     assert not ev["fails"], ev["fails"][:5]
     first = model.shape.first_candidate
+    score_err = 0.0
     for t in range(S):
         g = rec[t]
-        np.testing.assert_allclose(g["scores"], ev["scores"][t], rtol=0, atol=P.ROUTE_MARGIN / 4)
+        # within half the near-tie margin, two scores cannot swap across a gap
+        # of at least the margin
+        np.testing.assert_allclose(g["scores"], ev["scores"][t], rtol=0, atol=P.ROUTE_MARGIN / 2)
+        score_err = max(score_err, float(np.max(np.abs(g["scores"] - ev["scores"][t]))))
         np.testing.assert_array_equal(g["mask"].sum(1), np.asarray(ev["k"][t]) + 1 + first)
         rows = T.O.compaction(ev["sel"][t], L, first)
         for l in range(L):
@@ -104,5 +108,5 @@ def test_fullsize_trajectory_parity(w, sampled):
                 else:
                     assert not gk.any() and not gv.any(), (l, i, t)
     print(f"{w.name}: {S} steps, sampled {sampled}: worst hidden max rel err {worst:.3e}, "
-          f"worst K/V {kv_err:.3e}, adopted near-ties {ev['adopted']}")
+          f"worst K/V {kv_err:.3e}, worst score {score_err:.3e}, adopted near-ties {ev['adopted']}")
     assert kv_err < P.KV_TOL[s.dtype]

@@ -48,8 +48,10 @@ def build(w: Workload, device="cuda", extra_steps: int = 8, max_batch: Optional[
     dm = {k: mv(v) for k, v in synth.dm_weights(s, w.seed, gd).items()}
     pr = mv(synth.prior(s, w.seed, gd)) if prior else None
     ctx.buddy_set_weights(layers, dm, prior=pr, omega=omega if prior else 0.0)
+    if s.predictor_hidden > 0:
+        ctx.buddy_set_budget_predictor({k: mv(v) for k, v in synth.predictor_weights(s, w.seed, gd).items()})
     ctx.buddy_set_options(use_graph)
-    kv = pkg.KVCache(s.n_layers, s.n_kv_heads, s.head_dim, caps.tolist(), dt, device)
+    kv = pkg.KVCache(s.n_layers, s.n_kv_heads, s.head_dim, caps.tolist(), dt, device, masked=s.skip_kv == "masked")
     prefill(ctx, kv, w, ctxs, device, gd)
     k = torch.tensor(w.budgets(), dtype=torch.int32, device=device)
     return DeviceWorkload(w, ctx, kv, layers, dm, k, ctxs, caps, pr)
