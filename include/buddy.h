@@ -269,6 +269,28 @@ BUDDY_API int buddy_decode_step(buddy_ctx* ctx, const buddy_kv_state* kv, int32_
                       const int32_t* k, float* h_out, uint8_t* mask_out, int32_t* rows_out,
                       int32_t* count_out, float* scores_out, void* stream);
 
+/* Routed prefill of one prompt per sequence (Sec. 4.1; App. E "Prefill vs.
+ * Decode"), bf16 contexts created with max_prefill_tokens > 0.
+ * n_tok: HOST [batch] prompt lengths (>= 1, sum <= max_prefill_tokens);
+ * x: device [sum n_tok, d] fp32, the prompts' input hidden states, sequence
+ * by sequence (rows off_i .. off_i + n_tok[i] - 1 for sequence i, off_i the
+ * sum of the earlier lengths); k: device [batch] budgets as in
+ * buddy_decode_step; h_out: device [sum n_tok, d] fp32, every token's hidden
+ * state after the last block (must not alias x).  Optional device outputs:
+ * mask_out [batch, L] uint8, scores_out [batch, n_cand] fp32.
+ * Sequence i's tokens take positions len[i] .. len[i] + n_tok[i] - 1.  Blocks
+ * 0..c run on every token with causal attention; each sequence is routed once
+ * from its pooled context-layer cache (prompt included) and its last token's
+ * state after block c; each routed block runs on all tokens of the sequences
+ * that selected it; a skipped block stores zero K/V at every prompt position
+ * (BUDDY_SKIP_MASKED: nothing).  Then len[i] += n_tok[i].  The call
+ * synchronises `stream` once, after the routing, to size the later launches;
+ * it returns BUDDY_ERR_DEVICE (nothing written) when the device checks of
+ * buddy_decode_step fail (budgets, len[i] + n_tok[i] <= cap[i], <= max_pos). */
+BUDDY_API int buddy_prefill(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t batch, const int32_t* n_tok,
+                            const float* x, const int32_t* k, float* h_out, uint8_t* mask_out,
+                            float* scores_out, void* stream);
+
 /* buddy_decode_step with HOST buffers: h_in_host [batch, d] fp32, k_host
  * [batch] int32, h_out_host [batch, d] fp32, mask_host [batch, L] uint8 (or
  * NULL).  Copies the inputs to device staging buffers, runs the step, copies
@@ -299,6 +321,9 @@ enum {
   BUDDY_PROF_ROUTE, BUDDY_PROF_COMPACT, BUDDY_PROF_OTHER,
   BUDDY_PROF_GEMM_FIXUP,   /* split-K sums + epilogues of the GEMMs (larger batches) */
   BUDDY_PROF_ATTN_MERGE,   /* span merge of the tensor-core attention */
+  BUDDY_PROF_PF_GEMM,      /* prefill: projections (tcgen05, M-tiled) */
+  BUDDY_PROF_PF_ATTENTION, /* prefill: causal attention */
+  BUDDY_PROF_PF_OTHER,     /* prefill: RMSNorm, zero fill, advance */
   BUDDY_PROF_NCLASS
 };
 

@@ -22,10 +22,10 @@ EXPORTED = ["buddy_create", "buddy_destroy", "buddy_set_weights", "buddy_kv_appe
             "buddy_decode_step", "buddy_decode_step_host", "buddy_set_options",
             "buddy_device_status", "buddy_budget_to_k", "buddy_error_string", "buddy_version",
             "buddy_set_profiling", "buddy_profile_read", "buddy_profile_class_name",
-            "buddy_route_noalloc", "buddy_set_budget_predictor", "buddy_get_paths"]
+            "buddy_route_noalloc", "buddy_set_budget_predictor", "buddy_get_paths", "buddy_prefill"]
 PROF_CLASSES = ["check", "rmsnorm", "gemm_qkv", "qkv_finalize", "attention", "gemm_o", "gemm_gate_up",
                 "gemm_down", "route", "compact", "other", "gemm_fixup",
-                "attn_merge"]
+                "attn_merge", "pf_gemm", "pf_attention", "pf_other"]
 
 c_p = ctypes.c_void_p
 c_i32 = ctypes.c_int32
@@ -105,6 +105,9 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.buddy_set_budget_predictor.restype = ctypes.c_int
     lib.buddy_get_paths.argtypes = [c_p, ctypes.POINTER(c_i32), c_i32]
     lib.buddy_get_paths.restype = ctypes.c_int
+    lib.buddy_prefill.argtypes = [c_p, ctypes.POINTER(buddy_kv_state), c_i32, ctypes.POINTER(c_i32), c_p, c_p, c_p,
+                                  c_p, c_p, c_p]
+    lib.buddy_prefill.restype = ctypes.c_int
     for name in ("buddy_create", "buddy_set_weights", "buddy_kv_append", "buddy_route", "buddy_decode_step",
                  "buddy_decode_step_host", "buddy_set_options", "buddy_device_status", "buddy_set_profiling",
                  "buddy_profile_read"):
@@ -292,6 +295,14 @@ class Context:
                                           _ptr(k), _ptr(h_out), _ptr(mask_out), _ptr(rows_out),
                                           _ptr(count_out), _ptr(scores_out), _stream(stream)),
                "buddy_decode_step")
+
+    def buddy_prefill(self, kv: KVCache, n_tok: Sequence[int], x: torch.Tensor, k: torch.Tensor,
+                      h_out: torch.Tensor, mask_out=None, scores_out=None, stream=None):
+        """Routed prefill: x / h_out [sum(n_tok), d] fp32 device, n_tok host lengths."""
+        nt = (c_i32 * len(n_tok))(*[int(v) for v in n_tok])
+        _check(self.lib.buddy_prefill(self.handle, ctypes.byref(kv.state), len(n_tok), nt, _ptr(x), _ptr(k),
+                                      _ptr(h_out), _ptr(mask_out), _ptr(scores_out), _stream(stream)),
+               "buddy_prefill")
 
     def buddy_decode_step_host(self, kv: KVCache, h_in_host: torch.Tensor, k_host: torch.Tensor,
                                h_out_host: torch.Tensor, mask_host=None, stream=None):

@@ -55,7 +55,9 @@ static void free_ctx(buddy_ctx* x) {
   void* ptrs[] = {c.rope_cos, c.rope_sin, c.status, c.xn, c.act, c.attn_out, c.qkv, c.q,
                   c.attn_m, c.attn_l, c.attn_acc, c.attn_ctr, c.dm_u, c.mask, c.sel, c.scores, c.rows,
                   c.count, c.h_in_stage, c.h_out_stage, c.k_stage, c.mask_stage, c.xn_lo, c.act_lo, c.attn_lo,
-                  c.gemm_ws, c.gemm_ctr, c.attn_meta};
+                  c.gemm_ws, c.gemm_ctr, c.attn_meta, c.pf_xn, c.pf_xn_lo, c.pf_q, c.pf_attn, c.pf_attn_lo,
+                  c.pf_act, c.pf_act_lo, c.pf_tok_seq, c.pf_tok_t, c.pf_tok_pos, c.pf_rows, c.pf_items,
+                  c.pf_n_tok, c.pf_tok_end, c.pf_cnt, c.pf_hlast};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   if (x->cap_stream) cudaStreamDestroy(x->cap_stream);
@@ -146,6 +148,20 @@ extern "C" int buddy_create(const buddy_config* cfg, buddy_ctx** out) {
       (e = cudaMemset(c.attn_ctr, 0, B * c.nkv * sizeof(int32_t))) != cudaSuccess)
     return fail(e);
   c.dm_u_cols = c.r;
+  c.pf_max = g.max_prefill_tokens;
+  if (c.pf_max > 0) {
+    const size_t T = c.pf_max;
+    c.pf_items_max = (int64_t)(T / 64 + B) * c.nq;
+    if ((e = cudaMalloc(&c.pf_xn, T * c.d * c.esz)) || (e = cudaMalloc(&c.pf_xn_lo, T * c.d * c.esz)) ||
+        (e = dalloc(&c.pf_q, T * c.qd)) || (e = cudaMalloc(&c.pf_attn, T * c.qd * c.esz)) ||
+        (e = cudaMalloc(&c.pf_attn_lo, T * c.qd * c.esz)) || (e = cudaMalloc(&c.pf_act, T * c.F * c.esz)) ||
+        (e = cudaMalloc(&c.pf_act_lo, T * c.F * c.esz)) || (e = dalloc(&c.pf_tok_seq, T)) ||
+        (e = dalloc(&c.pf_tok_t, T)) || (e = dalloc(&c.pf_tok_pos, T)) ||
+        (e = dalloc(&c.pf_rows, (size_t)c.L * T)) ||
+        (e = dalloc(&c.pf_items, (size_t)(c.L + 1) * c.pf_items_max)) || (e = dalloc(&c.pf_n_tok, B)) ||
+        (e = dalloc(&c.pf_tok_end, B)) || (e = dalloc(&c.pf_cnt, B)) || (e = dalloc(&c.pf_hlast, B * c.d)))
+      return fail(e);
+  }
   if ((e = cudaStreamCreateWithFlags(&x->cap_stream, cudaStreamNonBlocking)) != cudaSuccess) return fail(e);
   launch_rope_table(c.rope_cos, c.rope_sin, c.max_pos, c.hd, (double)g.rope_theta, x->cap_stream);
   if ((e = cudaGetLastError()) != cudaSuccess || (e = cudaStreamSynchronize(x->cap_stream)) != cudaSuccess)
@@ -236,39 +252,6 @@ extern "C" int buddy_device_status(buddy_ctx* ctx, void* stream, int32_t* flags)
   return h[0] ? BUDDY_ERR_DEVICE : BUDDY_OK;
 }
 
-// ---------------------------------------------------------------------------
-// Profiler: an event pair around each launch group (direct-launch mode only).
-// ---------------------------------------------------------------------------
-static cudaEvent_t take_event(Ctx& c) {
-  if (c.ev_used == c.ev_pool.size()) {
-    cudaEvent_t e = nullptr;
-    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
-    c.ev_pool.push_back(e);
-  }
-  return c.ev_pool[c.ev_used++];
-}
-
-struct ProfScope {
-  Ctx& c;
-  cudaStream_t s;
-  Ctx::ProfRec rec{};
-  bool on;
-  ProfScope(Ctx& c_, cudaStream_t s_, int cls, int launches, bool on_) : c(c_), s(s_), on(on_) {
-    if (!on) return;
-    rec.cls = cls;
-    rec.launches = launches;
-    rec.a = take_event(c);
-    rec.b = take_event(c);
-    on = rec.a && rec.b;
-    if (on) cudaEventRecord(rec.a, s);
-  }
-  ~ProfScope() {
-    if (!on) return;
-    cudaEventRecord(rec.b, s);
-    c.prof.push_back(rec);
-  }
-};
-
 extern "C" int buddy_get_paths(buddy_ctx* ctx, int32_t* paths, int32_t n) {
   if (!ctx || !paths || n < 0 || n > 4) return BUDDY_ERR_ARG;
   const Ctx& c = ctx->c;
@@ -289,7 +272,7 @@ extern "C" const char* buddy_profile_class_name(int32_t cls) {
   static const char* names[BUDDY_PROF_NCLASS] = {"check", "rmsnorm", "gemm_qkv", "qkv_finalize",
                                                  "attention", "gemm_o", "gemm_gate_up", "gemm_down",
                                                  "route", "compact", "other", "gemm_fixup",
-                                                 "attn_merge"};
+                                                 "attn_merge", "pf_gemm", "pf_attention", "pf_other"};
   return (cls >= 0 && cls < BUDDY_PROF_NCLASS) ? names[cls] : "unknown";
 }
 
@@ -551,6 +534,25 @@ extern "C" int buddy_decode_step_host(buddy_ctx* ctx, const buddy_kv_state* kv, 
   if (mask_host) CK(cudaMemcpyAsync(mask_host, c.mask_stage, (size_t)batch * c.L, cudaMemcpyDeviceToHost, s));
   CK(cudaStreamSynchronize(s));
   return BUDDY_OK;
+}
+
+extern "C" int buddy_prefill(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t batch, const int32_t* n_tok,
+                             const float* x, const int32_t* k, float* h_out, uint8_t* mask_out, float* scores_out,
+                             void* stream) {
+  if (!ctx) return BUDDY_ERR_ARG;
+  Ctx& c = ctx->c;
+  if (!c.have_weights) return BUDDY_ERR_STATE;
+  if (c.pf_max <= 0 || c.dtype != BUDDY_DTYPE_BF16) return BUDDY_ERR_STATE;
+  if (batch < 1 || batch > c.maxB || !n_tok || !x || !k || !h_out || x == h_out) return BUDDY_ERR_ARG;
+  int rc = check_kv(c, kv, batch);
+  if (rc) return rc;
+  int64_t T = 0;
+  for (int i = 0; i < batch; ++i) {
+    if (n_tok[i] < 1) return BUDDY_ERR_RANGE;
+    T += n_tok[i];
+  }
+  if (T > c.pf_max) return BUDDY_ERR_RANGE;
+  return run_prefill(c, *kv, batch, n_tok, x, k, h_out, mask_out, scores_out, (cudaStream_t)stream);
 }
 
 extern "C" int buddy_route(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t batch, const float* h1,

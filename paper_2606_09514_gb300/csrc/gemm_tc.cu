@@ -466,6 +466,18 @@ int gemm_tc_prepare(Ctx& c) {
   // that would finish it (m x 256 fp32 per split): a fixup kernel spreads
   // them over all SMs.
   c.tc_defer = c.maxB > kTcDeferRows;
+  if (c.pf_max > 0) {
+    // prefill activations: 128-row boxes (one M-tile per copy)
+    if (!make_map(&c.pf_tmaps[0], c.pf_xn, c.pf_max, c.d, 128) ||
+        !make_map(&c.pf_tmaps[1], c.pf_attn, c.pf_max, c.qd, 128) ||
+        !make_map(&c.pf_tmaps[2], c.pf_act, c.pf_max, c.F, 128) ||
+        !make_map(&c.pf_tmaps[3], c.pf_xn_lo, c.pf_max, c.d, 128) ||
+        !make_map(&c.pf_tmaps[4], c.pf_attn_lo, c.pf_max, c.qd, 128) ||
+        !make_map(&c.pf_tmaps[5], c.pf_act_lo, c.pf_max, c.F, 128))
+      return BUDDY_ERR_CUDA;
+    const int rc = gemm_pf_prepare(c);
+    if (rc != BUDDY_OK) return rc;
+  }
   const cudaFuncAttribute A = cudaFuncAttributeMaxDynamicSharedMemorySize;
   const int qs0 = std::max(c.tc_smem[0], c.tc_panel ? c.tc_psmem[0] : 0);
   const int qs1 = std::max(c.tc_smem[1], c.tc_panel ? c.tc_psmem[1] : 0);

@@ -69,6 +69,25 @@ struct GemmArgs {
 
 struct Ctx;
 
+// Epilogue pointers of a prefill GEMM (gemm_pf.cu); unused ones stay null.
+struct PfEpi {
+  const int32_t* rows;      // compact row -> token row (nullptr: identity)
+  const float* resid_src;
+  float* resid_dst;
+  void* out_act;
+  void* out_act_lo;
+  float* q_out;
+  const float* bias;
+  const int32_t* tok_seq;
+  const int32_t* tok_pos;
+  const int32_t* len;
+  const int32_t* cache_len;
+  const int64_t* seq_off;
+  const int32_t* cap;
+  void* kc;
+  void* vc;
+};
+
 // Launch with programmatic stream serialisation when `pdl` is set (the kernel
 // then overlaps its prologue with the predecessor and synchronises with
 // pdl_wait()).
@@ -121,6 +140,17 @@ void launch_pool_refresh(const Ctx& c, const buddy_kv_state& kv, int n_seq, cons
 void launch_gemm_simt(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s);
 bool gemm_tc_supported(const Ctx& c);
 void launch_gemm_tc(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s);
+// prefill (gemm_pf.cu, attn_pf.cu, prefill.cu)
+int gemm_pf_prepare(Ctx& c);
+void launch_gemm_pf(const Ctx& c, int epi, bool split, int layer, int which, int xi, int m, const PfEpi& e,
+                    cudaStream_t s);
+void launch_attention_pf(const Ctx& c, int n_items, const int4* items, const int32_t* n_tok, const int32_t* base,
+                         const buddy_kv_state& kv, int layer, const float* q, void* out, void* out_lo,
+                         cudaStream_t s);
+void launch_pool_refresh_n(const Ctx& c, const buddy_kv_state& kv, int n_seq, const int32_t* n_new,
+                           cudaStream_t s);
+int run_prefill(Ctx& c, const buddy_kv_state& kv, int B, const int32_t* n_tok_host, const float* x,
+                const int32_t* k, float* h_out, uint8_t* mask_out, float* scores_out, cudaStream_t s);
 void launch_gemm_fix(const Ctx& c, int epi, const GemmArgs& a, cudaStream_t s);   // with c.tc_defer
 
 struct Ctx {
@@ -192,6 +222,28 @@ struct Ctx {
   // per GEMM sums the partials and applies the epilogue on every SM
   bool tc_defer = false;
 
+  // prefill scratch (max_prefill_tokens rows)
+  int pf_max = 0;
+  int64_t pf_items_max = 0;       // attention work items per block
+  void* pf_xn = nullptr;          // [pf_max, d] bf16, and its remainder term
+  void* pf_xn_lo = nullptr;
+  float* pf_q = nullptr;          // [pf_max, qd]
+  void* pf_attn = nullptr;        // [pf_max, qd] bf16 (+ remainder)
+  void* pf_attn_lo = nullptr;
+  void* pf_act = nullptr;         // [pf_max, F] bf16 (+ remainder)
+  void* pf_act_lo = nullptr;
+  int32_t* pf_tok_seq = nullptr;  // [pf_max] token row -> sequence
+  int32_t* pf_tok_t = nullptr;    // [pf_max] token row -> index in its prompt
+  int32_t* pf_tok_pos = nullptr;  // [pf_max] token row -> position
+  int32_t* pf_rows = nullptr;     // [L, pf_max] row lists of the routed blocks
+  int4* pf_items = nullptr;       // [(L + 1) * pf_items_max] attention work items
+  int32_t* pf_n_tok = nullptr;    // [maxB]
+  int32_t* pf_tok_end = nullptr;  // [maxB] one past the last token row of each prompt
+  int32_t* pf_cnt = nullptr;      // [maxB] positions the pooled context covers
+  float* pf_hlast = nullptr;      // [maxB, d] last prompt token's hidden state
+  CUtensorMap pf_tmaps[6];        // pf_xn, pf_attn, pf_act, then their remainder terms
+  int pf_stages[2] = {1, 1}, pf_smem[2] = {0, 0};
+
   // profiler: event pairs around kernel launches (direct-launch mode only)
   int profiling = 0;
   struct ProfRec { int cls; int launches; cudaEvent_t a, b; };
@@ -207,6 +259,39 @@ struct Ctx {
     bool operator<(const GraphKey& o) const;
   };
   std::map<GraphKey, cudaGraphExec_t> graphs;
+};
+
+// ---------------------------------------------------------------------------
+// Profiler: an event pair around each launch group (direct-launch mode only).
+// ---------------------------------------------------------------------------
+inline cudaEvent_t take_event(Ctx& c) {
+  if (c.ev_used == c.ev_pool.size()) {
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    c.ev_pool.push_back(e);
+  }
+  return c.ev_pool[c.ev_used++];
+}
+
+struct ProfScope {
+  Ctx& c;
+  cudaStream_t s;
+  Ctx::ProfRec rec{};
+  bool on;
+  ProfScope(Ctx& c_, cudaStream_t s_, int cls, int launches, bool on_) : c(c_), s(s_), on(on_) {
+    if (!on) return;
+    rec.cls = cls;
+    rec.launches = launches;
+    rec.a = take_event(c);
+    rec.b = take_event(c);
+    on = rec.a && rec.b;
+    if (on) cudaEventRecord(rec.a, s);
+  }
+  ~ProfScope() {
+    if (!on) return;
+    cudaEventRecord(rec.b, s);
+    c.prof.push_back(rec);
+  }
 };
 
 // Positions layer l holds for each sequence (where its next entry goes):

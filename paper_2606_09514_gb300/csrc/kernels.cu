@@ -552,20 +552,20 @@ __global__ void __launch_bounds__(256) kv_append_kernel(int n_new, int nkv, int 
 }
 
 template <typename T>
-__global__ void __launch_bounds__(256) pool_refresh_kernel(int n_new, int nkv, int hd, int feature,
-                                                           const int32_t* ids, const int32_t* len,
+__global__ void __launch_bounds__(256) pool_refresh_kernel(int n_new, const int32_t* n_new_of, int nkv, int hd,
+                                                           int feature, const int32_t* ids, const int32_t* len,
                                                            const int64_t* seq_off,
                                                            const int32_t* cap, const T* K0, const T* V0,
                                                            float* pool, const int32_t* status) {
   pdl_wait();
   pdl_trigger();
   if (call_aborted(status)) return;
-  const int s = ids[blockIdx.y];
+  const int s = ids ? ids[blockIdx.y] : blockIdx.y;
   const int kvd = nkv * hd;
   const int x = blockIdx.x * blockDim.x + threadIdx.x;
   if (x >= kvd) return;
   const int g = x / hd, e = x - g * hd;
-  const int n = len[s] + n_new;
+  const int n = len[s] + (n_new_of ? n_new_of[s] : n_new);
   const int64_t off = kv_offset(seq_off, cap, s, nkv, hd, g, 0) + e;
   float acc = 0.f;
   for (int p = 0; p < n; ++p) {
@@ -599,11 +599,28 @@ void launch_pool_refresh(const Ctx& c, const buddy_kv_state& kv, int n_seq, cons
   const int l = c.cl;
   const int32_t* base = cache_len(c, kv, l);
   if (c.dtype == BUDDY_DTYPE_BF16)
-    pool_refresh_kernel<bf16><<<g, 256, 0, s>>>(n_new, c.nkv, c.hd, c.feature, ids, base, kv.seq_off, kv.cap,
-                                                (const bf16*)kv.k_cache[l], (const bf16*)kv.v_cache[l],
+    pool_refresh_kernel<bf16><<<g, 256, 0, s>>>(n_new, nullptr, c.nkv, c.hd, c.feature, ids, base, kv.seq_off,
+                                                kv.cap, (const bf16*)kv.k_cache[l], (const bf16*)kv.v_cache[l],
                                                 kv.pool_sum, c.status);
   else
-    pool_refresh_kernel<float><<<g, 256, 0, s>>>(n_new, c.nkv, c.hd, c.feature, ids, base, kv.seq_off,
+    pool_refresh_kernel<float><<<g, 256, 0, s>>>(n_new, nullptr, c.nkv, c.hd, c.feature, ids, base, kv.seq_off,
+                                                 kv.cap, (const float*)kv.k_cache[l],
+                                                 (const float*)kv.v_cache[l], kv.pool_sum, c.status);
+}
+
+// Pooled context of sequences 0..n_seq-1 recomputed over their first
+// base + n_new[s] positions of the context layer (prefill).
+void launch_pool_refresh_n(const Ctx& c, const buddy_kv_state& kv, int n_seq, const int32_t* n_new,
+                           cudaStream_t s) {
+  dim3 g((c.kvd + 255) / 256, n_seq);
+  const int l = c.cl;
+  const int32_t* base = cache_len(c, kv, l);
+  if (c.dtype == BUDDY_DTYPE_BF16)
+    pool_refresh_kernel<bf16><<<g, 256, 0, s>>>(0, n_new, c.nkv, c.hd, c.feature, nullptr, base, kv.seq_off,
+                                                kv.cap, (const bf16*)kv.k_cache[l], (const bf16*)kv.v_cache[l],
+                                                kv.pool_sum, c.status);
+  else
+    pool_refresh_kernel<float><<<g, 256, 0, s>>>(0, n_new, c.nkv, c.hd, c.feature, nullptr, base, kv.seq_off,
                                                  kv.cap, (const float*)kv.k_cache[l],
                                                  (const float*)kv.v_cache[l], kv.pool_sum, c.status);
 }

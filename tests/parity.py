@@ -84,3 +84,35 @@ def max_rel_err(g: np.ndarray, o: np.ndarray) -> float:
 def sel_from_mask(mask: np.ndarray, first: int = 1) -> List[List[int]]:
     L = mask.shape[1]
     return [[l for l in range(first, L - 1) if mask[i, l]] for i in range(mask.shape[0])]
+
+
+def oracle_for(dw, gen_device="cuda"):
+    """Oracle model and state of a device workload (tests/GPU only)."""
+    from oracle import adapter as A
+    from workloads import synth
+    w = dw.w
+    s = w.shape
+    model = A.build_model(s, w.seed, layer_source=lambda l: synth.layer_weights(s, w.seed, l, gen_device),
+                          dm_source=lambda: synth.dm_weights(s, w.seed, gen_device),
+                          prior=dw.prior, omega=0.1 if dw.prior is not None else 0.0,
+                          cache_layers=s.n_layers,
+                          predictor_source=lambda: synth.predictor_weights(s, w.seed, gen_device))
+    st = A.build_state(s, w.seed, w.contexts(), gen_device=gen_device)
+    return model, st
+
+
+def adopt(model, rr, g_mask, k_given):
+    """Near-tie rules: the oracle takes the GPU's budget where the Budget
+    Predictor's argmax is a near-tie, then the GPU's set where the layer
+    ranking is.  Returns (sets, budgets, failures, adopted)."""
+    from oracle import buddy_oracle as O
+    first = model.shape.first_candidate
+    g_sel = sel_from_mask(g_mask, first)
+    g_k = [len(x) for x in g_sel]
+    logits = [O.predictor_logits(model.predictor, rr.x[i]) if model.predictor is not None else None
+              for i in range(len(g_sel))]
+    ks, fails_k = adopt_budgets(rr.k, g_k, logits, k_given)
+    o_sel = [rr.sel[i] if ks[i] == rr.k[i] else O.top_k_layers(rr.scores[i], ks[i], first)
+             for i in range(len(ks))]
+    sel, fails, n = adopt_routes(rr.scores, o_sel, g_sel, ks, first)
+    return sel, ks, fails_k + fails, n

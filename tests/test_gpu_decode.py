@@ -19,37 +19,9 @@ from workloads import synth
 pytestmark = pytest.mark.gpu
 
 
-def _oracle_for(dw, gen_device="cuda"):
-    w = dw.w
-    s = w.shape
-    model = A.build_model(s, w.seed, layer_source=lambda l: synth.layer_weights(s, w.seed, l, gen_device),
-                          dm_source=lambda: synth.dm_weights(s, w.seed, gen_device),
-                          prior=dw.prior, omega=0.1 if dw.prior is not None else 0.0,
-                          cache_layers=s.n_layers,
-                          predictor_source=lambda: synth.predictor_weights(s, w.seed, gen_device))
-    st = A.build_state(s, w.seed, w.contexts(), gen_device=gen_device)
-    return model, st
-
-
-def adopt(model, rr, g_mask, k_given):
-    """Near-tie rules: the oracle takes the GPU's budget where the Budget
-    Predictor's argmax is a near-tie, then the GPU's set where the layer
-    ranking is.  Returns (sets, budgets, failures, adopted)."""
-    first = model.shape.first_candidate
-    g_sel = P.sel_from_mask(g_mask, first)
-    g_k = [len(x) for x in g_sel]
-    logits = [O.predictor_logits(model.predictor, rr.x[i]) if model.predictor is not None else None
-              for i in range(len(g_sel))]
-    ks, fails_k = P.adopt_budgets(rr.k, g_k, logits, k_given)
-    o_sel = [rr.sel[i] if ks[i] == rr.k[i] else O.top_k_layers(rr.scores[i], ks[i], first)
-             for i in range(len(ks))]
-    sel, fails, n = P.adopt_routes(rr.scores, o_sel, g_sel, ks, first)
-    return sel, ks, fails_k + fails, n
-
-
 def run_parity(w, steps=None, use_graph=False, prior=False, check_kv=True):
     dw = D.build(w, use_graph=use_graph, prior=prior)
-    model, st = _oracle_for(dw)
+    model, st = P.oracle_for(dw)
     s = w.shape
     B, L, Lm = w.batch, s.n_layers, s.n_cand
     masked = s.skip_kv == "masked"
@@ -74,7 +46,7 @@ def run_parity(w, steps=None, use_graph=False, prior=False, check_kv=True):
         info = {}
 
         def override(rr):
-            sel, ks, fails, n = adopt(model, rr, g_mask, k)
+            sel, ks, fails, n = P.adopt(model, rr, g_mask, k)
             info["fails"], info["n"], info["k"] = fails, n, ks
             return sel
 
@@ -208,7 +180,7 @@ def test_route_entry_point_matches_oracle_router():
     dw.ctx.buddy_route(dw.kv, h1, dw.k, sel, mask, sc)
     torch.cuda.synchronize()
     assert dw.ctx.buddy_device_status() == 0
-    model, _ = _oracle_for(dw)
+    model, _ = P.oracle_for(dw)
     sh = model.shape
     lens = dw.kv.len.cpu().numpy()
     o_sel, o_sc = [], []

@@ -31,7 +31,7 @@ class DeviceWorkload:
 
 def build(w: Workload, device="cuda", extra_steps: int = 8, max_batch: Optional[int] = None,
           prior: bool = False, omega: float = 0.1, use_graph: bool = False,
-          gen_device: Optional[str] = None) -> DeviceWorkload:
+          gen_device: Optional[str] = None, max_prefill_tokens: int = 0) -> DeviceWorkload:
     """gen_device: where the generator runs ("cpu": every tensor is drawn on
     the host and copied to `device` once; default: on `device`)."""
     import paper_2606_09514_gb300 as pkg
@@ -42,7 +42,8 @@ def build(w: Workload, device="cuda", extra_steps: int = 8, max_batch: Optional[
     mv = lambda t: t.to(device)
     ctxs = w.contexts()
     caps = ctxs + w.steps + extra_steps + 1
-    ctx = pkg.Context.for_shape(s, max_batch=max_batch or w.batch, max_pos=int(caps.max()))
+    ctx = pkg.Context.for_shape(s, max_batch=max_batch or w.batch, max_pos=int(caps.max()),
+                                max_prefill_tokens=max_prefill_tokens)
     layers = [pkg.pack_layer({k: mv(v) for k, v in synth.layer_weights(s, w.seed, l, gd).items()})
               for l in range(s.n_layers)]
     dm = {k: mv(v) for k, v in synth.dm_weights(s, w.seed, gd).items()}

@@ -184,5 +184,17 @@ def h_in(shape: ModelShape, seed: int, step: int, seqs: Sequence[int], device="c
     return out
 
 
+def prompt_inputs(shape: ModelShape, seed: int, lengths: Sequence[int], device="cpu") -> torch.Tensor:
+    """Input hidden states of one prompt per sequence, [sum(lengths), d] fp32
+    N(0,1), sequence by sequence; one stream per (sequence, token)."""
+    out = torch.empty(int(sum(lengths)), shape.d_model, dtype=torch.float32, device=device)
+    r = 0
+    for i, n in enumerate(lengths):
+        for t in range(int(n)):
+            fill_normal_(out[r], stream_key(seed, "h_in", 1 << 20 | i, t), 1.0)
+            r += 1
+    return out
+
+
 def workload_h_in(w: Workload, step: int, device="cpu") -> torch.Tensor:
     return h_in(w.shape, w.seed, step, range(w.batch), device)
