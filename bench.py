@@ -39,6 +39,15 @@ METRIC = "budget-routed decode tokens/s at 1 GB300 per budget; % of HBM/tensor r
 NCU_TRAFFIC_PER_LAUNCH = {("llama3-8b-b1", "gemm_gate_up"): 238353664}
 DEFAULT_WORKLOAD = "llama3-8b-b1"
 PER_CONFIG = ["llama3-8b-b64-mixed", "llama2-13b-b32", "qwen2.5-7b-b256"]
+PREFILL_WORKLOAD = "llama3-8b-prefill-b16"
+
+
+def _peak_tflops_burst():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"])
+    except Exception:
+        return 1900.0
 
 
 def _peaks():
@@ -370,6 +379,79 @@ def measure(w, K, W, dev, ws, local, use_graph=True, e2e=True):
     return out
 
 
+def measure_prefill(w, K, W, dev, ws, local):
+    """Times K routed prefill calls of workload w's prompts (fresh sequences:
+    positions are reset before each call, as a server reuses a slot) after W
+    warm-up calls, then one profiled call for the kernel classes."""
+    import torch
+
+    from workloads import configs as C
+    from workloads import cost
+    from workloads import device as D
+    from workloads import synth
+
+    s = w.shape
+    lengths = [int(v) for v in C.prompt_lengths(w)]
+    T = int(sum(lengths))
+    dw = D.build(w, device=dev, extra_steps=max(lengths) + 2, max_prefill_tokens=T)
+    ctx, kv = dw.ctx, dw.kv
+    x = synth.prompt_inputs(s, w.seed, lengths, dev)
+    h_out = torch.empty(T, s.d_model, device=dev)
+    mask = torch.empty(w.batch, s.n_layers, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def call():
+        kv.len.zero_()
+        ctx.buddy_prefill(kv, lengths, x, dw.k, h_out, mask)
+
+    for _ in range(W):
+        call()
+    torch.cuda.synchronize(dev)
+    if ctx.buddy_device_status() != 0:
+        raise RuntimeError("device error flag during prefill warm-up")
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        _barrier(ws)
+        torch.cuda.synchronize(dev)
+        start.record(stream)
+        for _ in range(K):
+            call()
+        end.record(stream)
+        torch.cuda.synchronize(dev)
+        _barrier(ws)
+    ms = start.elapsed_time(end)
+    ms_max, value = aggregate(ms, T * K, ws, dev)
+    ctx.buddy_set_profiling(True)
+    ctx.buddy_profile_read()
+    call()
+    torch.cuda.synchronize(dev)
+    prof = ctx.buddy_profile_read()
+    ctx.buddy_set_profiling(False)
+    m = mask.cpu().numpy()
+    c = cost.prefill_cost(s, m, lengths, [0] * w.batch)
+    hbm, _, _ = _peaks()
+    burst = _peak_tflops_burst()
+    call_ms = ms_max / K
+    gemm_ms = prof["pf_gemm"][0]
+    out = {"workload": w.name, "value": round(value, 1), "unit": "tokens/s", "ms_per_call": round(call_ms, 3),
+           "calls": K, "warmup": W, "prompts": w.batch, "tokens_per_call": T,
+           "prompt_lengths": lengths, "k": w.k_args,
+           "tflops_per_call": round(c["flops"] / 1e12, 3),
+           "achieved_tflops": round(c["flops"] / (call_ms / 1e3) / 1e12, 1),
+           "roofline": {"bound": "tensor", "kernel": "pf_gemm",
+                        "achieved": round(c["gemm_flops"] / (gemm_ms / 1e3) / 1e12, 1) if gemm_ms > 0 else None,
+                        "peak": burst, "unit": "TFLOP/s",
+                        "frac": round(c["gemm_flops"] / (gemm_ms / 1e3) / 1e12 / burst, 4) if gemm_ms > 0 else None,
+                        "traffic": None, "flops_per_call": c["gemm_flops"], "peak_source": "measured bf16_tflops"},
+           "call_roofline_frac": round(max(c["flops"] / (burst * 1e12), c["bytes"] / (hbm * 1e9)) * 1e3 / call_ms, 4),
+           "kernel_ms_per_call": {k: round(v[0], 4) for k, v in prof.items() if v[1] > 0},
+           "paths": ctx.buddy_get_paths(), "clocks": clk.summary()}
+    ctx.close()
+    del dw, kv, ctx, x, h_out
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_ours(args, ws, rank, local):
     import torch
 
@@ -395,6 +477,8 @@ def run_ours(args, ws, rank, local):
             wc = C.BY_NAME[name]
             r = measure(wc, wc.steps, args.warmup, dev, ws, local, use_graph=not args.no_graph, e2e=False)
             out["per_config"][name] = r
+        # routed prefill (the paper's other speed column)
+        out["prefill"] = measure_prefill(C.BY_NAME[PREFILL_WORKLOAD], 5, 3, dev, ws, local)
     if rank == 0 and not args.no_cpu:
         o = oracle_sample(w, n_layers_sample=None, steps=1, device=dev)
         out["cpu_baseline"] = {"value": round(o["tokens"] / o["scaled_seconds"], 5), "unit": "tokens/s",

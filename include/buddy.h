@@ -314,6 +314,15 @@ BUDDY_API int buddy_set_options(buddy_ctx* ctx, int32_t use_graph);
  * paths[3] split-K sums in a separate fixup kernel (0/1).  n <= 4 entries. */
 BUDDY_API int buddy_get_paths(buddy_ctx* ctx, int32_t* paths, int32_t n);
 
+/* Limit of every bounded wait inside the tensor-core GEMM pipelines (TMA
+ * stages, MMA completion, accumulator hand-over), in nanoseconds; ns <= 0
+ * restores the default of 4 s.  A wait that runs out makes its kernel stop
+ * (after its copies and MMAs in flight have completed), raise
+ * BUDDY_DEV_TIMEOUT and leave its outputs incomplete; buddy_device_status
+ * then reports the bit and re-arms the kernels' arrival counters, so the
+ * context stays usable.  Synchronises the device; drops captured graphs. */
+BUDDY_API int buddy_set_wait_limit(buddy_ctx* ctx, int64_t ns);
+
 /* Kernel classes reported by the profiler. */
 enum {
   BUDDY_PROF_CHECK = 0, BUDDY_PROF_RMSNORM, BUDDY_PROF_GEMM_QKV, BUDDY_PROF_QKV_FINALIZE,

@@ -22,7 +22,8 @@ EXPORTED = ["buddy_create", "buddy_destroy", "buddy_set_weights", "buddy_kv_appe
             "buddy_decode_step", "buddy_decode_step_host", "buddy_set_options",
             "buddy_device_status", "buddy_budget_to_k", "buddy_error_string", "buddy_version",
             "buddy_set_profiling", "buddy_profile_read", "buddy_profile_class_name",
-            "buddy_route_noalloc", "buddy_set_budget_predictor", "buddy_get_paths", "buddy_prefill"]
+            "buddy_route_noalloc", "buddy_set_budget_predictor", "buddy_get_paths", "buddy_prefill",
+            "buddy_set_wait_limit"]
 PROF_CLASSES = ["check", "rmsnorm", "gemm_qkv", "qkv_finalize", "attention", "gemm_o", "gemm_gate_up",
                 "gemm_down", "route", "compact", "other", "gemm_fixup",
                 "attn_merge", "pf_gemm", "pf_attention", "pf_other"]
@@ -108,6 +109,8 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.buddy_prefill.argtypes = [c_p, ctypes.POINTER(buddy_kv_state), c_i32, ctypes.POINTER(c_i32), c_p, c_p, c_p,
                                   c_p, c_p, c_p]
     lib.buddy_prefill.restype = ctypes.c_int
+    lib.buddy_set_wait_limit.argtypes = [c_p, ctypes.c_int64]
+    lib.buddy_set_wait_limit.restype = ctypes.c_int
     for name in ("buddy_create", "buddy_set_weights", "buddy_kv_append", "buddy_route", "buddy_decode_step",
                  "buddy_decode_step_host", "buddy_set_options", "buddy_device_status", "buddy_set_profiling",
                  "buddy_profile_read"):
@@ -271,6 +274,9 @@ class Context:
                 "attention": "mma.sync tensor-core" if v[1] else "CUDA-core",
                 "rmsnorm": "inside the QKV and gate/up GEMMs" if v[2] else "separate kernel",
                 "split_k_fixup": "separate kernel" if v[3] else "last-arriving CTA"}
+
+    def buddy_set_wait_limit(self, ns: int):
+        _check(self.lib.buddy_set_wait_limit(self.handle, int(ns)), "buddy_set_wait_limit")
 
     def buddy_set_options(self, use_graph: bool):
         _check(self.lib.buddy_set_options(self.handle, 1 if use_graph else 0), "buddy_set_options")

@@ -223,6 +223,16 @@ extern "C" int buddy_set_budget_predictor(buddy_ctx* ctx, const buddy_predictor_
   return BUDDY_OK;
 }
 
+extern "C" int buddy_set_wait_limit(buddy_ctx* ctx, int64_t ns) {
+  if (!ctx) return BUDDY_ERR_ARG;
+  Ctx& c = ctx->c;
+  CK(cudaDeviceSynchronize());
+  c.wait_ns = ns > 0 ? (uint64_t)ns : 4000000000ull;
+  for (auto& kv : c.graphs) cudaGraphExecDestroy(kv.second);   // the limit is baked into captured launches
+  c.graphs.clear();
+  return BUDDY_OK;
+}
+
 extern "C" int buddy_set_options(buddy_ctx* ctx, int32_t use_graph) {
   if (!ctx) return BUDDY_ERR_ARG;
   ctx->c.use_graph = use_graph ? 1 : 0;
@@ -247,6 +257,11 @@ extern "C" int buddy_device_status(buddy_ctx* ctx, void* stream, int32_t* flags)
   CK(cudaMemcpyAsync(h, c.status, 2 * sizeof(int32_t), cudaMemcpyDeviceToHost, s));
   CK(cudaStreamSynchronize(s));
   CK(cudaMemsetAsync(c.status, 0, 2 * sizeof(int32_t), s));
+  if (h[0] & BUDDY_DEV_TIMEOUT) {
+    // a GEMM that gave up left split-K arrival counters mid-count: re-arm them
+    if (c.gemm_ctr) CK(cudaMemsetAsync(c.gemm_ctr, 0, c.gemm_ctr_n * sizeof(int32_t), s));
+    CK(cudaMemsetAsync(c.attn_ctr, 0, (size_t)c.maxB * c.nkv * sizeof(int32_t), s));
+  }
   CK(cudaStreamSynchronize(s));
   *flags = h[0];
   return h[0] ? BUDDY_ERR_DEVICE : BUDDY_OK;

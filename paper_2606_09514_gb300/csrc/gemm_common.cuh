@@ -97,6 +97,7 @@ struct TcParams {
   // Deferred fixup: units only stage their partials; a second kernel
   // (gemm_fix_kernel) sums the splits and applies the epilogue on every SM.
   int defer;
+  uint64_t wait_ns;       // limit of each pipeline wait (the drain waits keep kWaitLimitNs)
 };
 
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }

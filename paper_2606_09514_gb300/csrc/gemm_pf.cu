@@ -61,6 +61,7 @@ struct PfParams {
   bf16* vc;
   int nq, nkv, hd;
   int32_t* status;
+  uint64_t wait_ns;        // limit of each pipeline wait (the drain waits keep kWaitLimitNs)
 };
 
 template <int EPI>
@@ -234,7 +235,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x) {
         const int mt = u / p.n_tiles, nt = u - mt * p.n_tiles;
         for (int kb = 0; kb < p.kb_total; ++kb) {
-          if (!ptx::mbar_wait_bounded(&empty_bar[stage], ph ^ 1u, kWaitLimitNs, &abort_flag)) {
+          if (!ptx::mbar_wait_bounded(&empty_bar[stage], ph ^ 1u, p.wait_ns, &abort_flag)) {
             ok = false;
             break;
           }
@@ -268,11 +269,11 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       int n_consumed = 0;
       bool ok = true;
       for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x) {
-        if (!ptx::mbar_wait_bounded(&tempty_bar[acc], acc_ph ^ 1u, kWaitLimitNs, &abort_flag)) break;
+        if (!ptx::mbar_wait_bounded(&tempty_bar[acc], acc_ph ^ 1u, p.wait_ns, &abort_flag)) break;
         ptx::tc_fence_after();
         const uint32_t d = tmem_base + (uint32_t)acc * 256u;
         for (int kb = 0; kb < p.kb_total; ++kb) {
-          if (!ptx::mbar_wait_bounded(&full_bar[stage], ph, kWaitLimitNs, &abort_flag)) {
+          if (!ptx::mbar_wait_bounded(&full_bar[stage], ph, p.wait_ns, &abort_flag)) {
             ok = false;
             break;
           }
@@ -310,7 +311,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     int acc = 0;
     uint32_t acc_ph = 0;
     for (int u = blockIdx.x; u < p.units; u += gridDim.x) {
-      const bool ok = ptx::mbar_wait_bounded(&tfull_bar[acc], acc_ph, kWaitLimitNs, &abort_flag);
+      const bool ok = ptx::mbar_wait_bounded(&tfull_bar[acc], acc_ph, p.wait_ns, &abort_flag);
       if (epi_bar_any(!ok)) break;
       ptx::tc_fence_after();
       const int mt = u / p.n_tiles, nt = u - mt * p.n_tiles;
@@ -393,6 +394,7 @@ void launch_gemm_pf(const Ctx& c, int epi, bool split, int layer, int which, int
   p.nkv = c.nkv;
   p.hd = c.hd;
   p.status = c.status;
+  p.wait_ns = c.wait_ns;
   const CUtensorMap& tw = c.tmaps_host[(size_t)layer * 4 + which];
   const CUtensorMap& tx = c.pf_tmaps[xi];
   const CUtensorMap& txlo = c.pf_tmaps[3 + xi];

@@ -149,7 +149,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if (panel) ptx::mbar_arrive(&full_bar[stage]);
             else ptx::mbar_arrive_expect_tx(&full_bar[stage], x_bytes);
           } else {
-            if (!ptx::mbar_wait_bounded(&empty_bar[stage], ph ^ 1u, kWaitLimitNs, &abort_flag)) {
+            if (!ptx::mbar_wait_bounded(&empty_bar[stage], ph ^ 1u, p.wait_ns, &abort_flag)) {
               ok = false;
               break;
             }
@@ -184,15 +184,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x, ++ui) {
         const int split = u / p.n_tiles;
         const int kb0 = split * p.kb_per_split, kb1 = min(p.kb_total, kb0 + p.kb_per_split);
-        if (!ptx::mbar_wait_bounded(&tempty_bar[acc], acc_ph ^ 1u, kWaitLimitNs, &abort_flag)) break;
+        if (!ptx::mbar_wait_bounded(&tempty_bar[acc], acc_ph ^ 1u, p.wait_ns, &abort_flag)) break;
         if (panel &&
-            !ptx::mbar_wait_bounded(&pfull_bar[ui & 1], (uint32_t)((ui >> 1) & 1), kWaitLimitNs, &abort_flag))
+            !ptx::mbar_wait_bounded(&pfull_bar[ui & 1], (uint32_t)((ui >> 1) & 1), p.wait_ns, &abort_flag))
           break;
         ptx::tc_fence_after();
         const uint32_t d = tmem_base + (uint32_t)acc * acc_cols;
         const uint8_t* pan = smem + p.panel_off + (size_t)(ui & 1) * p.panel_bytes;
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!ptx::mbar_wait_bounded(&full_bar[stage], ph, kWaitLimitNs, &abort_flag)) {
+          if (!ptx::mbar_wait_bounded(&full_bar[stage], ph, p.wait_ns, &abort_flag)) {
             ok = false;
             break;
           }
@@ -251,7 +251,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         epi_bar();
         if (et == 0) ptx::mbar_arrive(&pfull_bar[(ui + 1) & 1]);
       }
-      const bool ok = ptx::mbar_wait_bounded(&tfull_bar[acc], acc_ph, kWaitLimitNs, &abort_flag);
+      const bool ok = ptx::mbar_wait_bounded(&tfull_bar[acc], acc_ph, p.wait_ns, &abort_flag);
       if (epi_bar_any(!ok)) break;
       ptx::tc_fence_after();
       tc_epilogue_unit<EPI, SPLIT>(p, u, m, tmem_base + (uint32_t)acc * acc_cols, &tempty_bar[acc], &last_flag);
@@ -553,6 +553,7 @@ static TcParams tc_params(const Ctx& c, const GemmArgs& a, size_t* smem_out) {
   }
   p.count_late = a.count_late ? 1 : 0;
   p.defer = c.tc_defer ? 1 : 0;
+  p.wait_ns = c.wait_ns;
   p.nq = c.nq;
   p.nkv = c.nkv;
   p.hd = c.hd;

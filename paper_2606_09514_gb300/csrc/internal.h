@@ -163,6 +163,7 @@ struct Ctx {
   size_t esz;
   int device, num_sms;
   bool pdl = true;             // programmatic dependent launch between step kernels
+  uint64_t wait_ns = 4000000000ull;   // limit of each bounded wait in the GEMM pipelines
 
   bool have_weights = false;
   std::vector<buddy_layer_weights> layers;

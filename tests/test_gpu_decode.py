@@ -241,6 +241,38 @@ def test_device_checks_write_nothing():
     assert not torch.all(h_out == 7.0)
 
 
+def test_gemm_wait_limit_runs_out_and_context_recovers():
+    """With a wait limit far below the time a TMA stage takes, the GEMMs give
+    up: the step reports BUDDY_DEV_TIMEOUT.  Restoring the limit, the same
+    step from the same state equals a fresh context's result (the arrival
+    counters were re-armed)."""
+    import paper_2606_09514_gb300 as pkg
+    for w in (C.T_GQA, C.scaled(C.T_QWEN, ctx=[5, 300, 64], k=[1, 3, 5], name="t-qwen-b3-timeout")):
+        s = w.shape
+        h_in = synth.workload_h_in(w, 0, "cuda")
+        ref = D.build(w)
+        h_ref = torch.empty(w.batch, s.d_model, device="cuda")
+        ref.ctx.buddy_decode_step(ref.kv, h_in, ref.k, h_ref)
+        torch.cuda.synchronize()
+        assert ref.ctx.buddy_device_status() == 0
+        dw = D.build(w)
+        len0, pool0 = dw.kv.len.clone(), dw.kv.pool_sum.clone()
+        h_out = torch.empty(w.batch, s.d_model, device="cuda")
+        dw.ctx.buddy_set_wait_limit(1)
+        dw.ctx.buddy_decode_step(dw.kv, h_in, dw.k, h_out)
+        torch.cuda.synchronize()
+        assert dw.ctx.buddy_device_status() & pkg.binding.BUDDY_DEV_TIMEOUT
+        dw.ctx.buddy_set_wait_limit(0)
+        dw.kv.len.copy_(len0)
+        dw.kv.pool_sum.copy_(pool0)
+        dw.ctx.buddy_decode_step(dw.kv, h_in, dw.k, h_out)
+        torch.cuda.synchronize()
+        assert dw.ctx.buddy_device_status() == 0
+        assert torch.equal(h_out, h_ref)
+        ref.ctx.close()
+        dw.ctx.close()
+
+
 def test_host_buffer_entry_matches_device_entry():
     w = C.T_GQA
     outs = []

@@ -212,6 +212,19 @@ P_QWEN_3L_B256 = Workload("qwen2.5-7b-3layer-b256",
                           batch=256, steps=8, seed=0, ctx_kind="lognormal", ctx_args=(2048, 0.5, 512, 8192),
                           k_kind="fixed", k_args=(1,))
 
+# Routed prefill: 16 prompts of 128..1024 tokens (seeded), fresh sequences,
+# budget k = 15 of 30 (the 50% column of the paper's speed table).
+PF_LLAMA3_B16 = Workload("llama3-8b-prefill-b16", LLAMA3_8B, batch=16, steps=1, seed=0,
+                         ctx_kind="fixed", ctx_args=(0,), k_kind="fixed", k_args=(15,),
+                         description="Llama-3-8B shape, bf16, 16 prompts of U[128,1024] tokens, k=15 of 30")
+
+
+def prompt_lengths(w: Workload, lo: int = 128, hi: int = 1024) -> np.ndarray:
+    """Seeded prompt lengths U[lo, hi] of a prefill workload."""
+    rng = np.random.default_rng(np.random.SeedSequence([w.seed, 0x7066]))
+    return rng.integers(lo, hi + 1, size=w.batch, dtype=np.int64)
+
+
 # Router variants on the small shapes: K and K + V planner features, a context
 # layer c > 0, the masked skip-KV variant, and the Budget Predictor (budget 0 =
 # predicted).
@@ -236,8 +249,8 @@ T_VARIANTS = [
              k_kind="list", k_args=(1, 2, 3, 3, 2, 1)),
 ]
 
-BY_NAME = {w.name: w for w in FULL_WORKLOADS + [T_GQA, T_QWEN, T_F32, T_PRED, P_LLAMA3_3L_B1, P_QWEN_3L_B256]
-           + T_VARIANTS}
+BY_NAME = {w.name: w for w in FULL_WORKLOADS + [T_GQA, T_QWEN, T_F32, T_PRED, P_LLAMA3_3L_B1, P_QWEN_3L_B256,
+                                                PF_LLAMA3_B16] + T_VARIANTS}
 
 
 def with_shape(w: Workload, name: Optional[str] = None, **shape_changes) -> Workload:

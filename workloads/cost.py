@@ -78,5 +78,28 @@ def step_cost(s: ModelShape, mask: np.ndarray, n_ctx: Sequence[int]) -> dict:
             "flops": flops, "exec_pairs": exec_pairs, "layers_used": int(used.sum())}
 
 
+def prefill_cost(s: ModelShape, mask: np.ndarray, lengths: Sequence[int], n0: Sequence[int]) -> dict:
+    """Algorithmic FLOPs and bytes of one routed prefill: every executed
+    (prompt, layer) pair runs its T_i tokens through the projections
+    (2 * layer_params FLOPs per token) and causal attention (token t attends
+    to n0_i + t + 1 positions: 4 * n_q * hd FLOPs per position); bytes are
+    the union of executed layers' weights, the K/V written and read once,
+    and the hidden states in and out."""
+    mask = np.asarray(mask, dtype=bool)
+    B, L = mask.shape
+    T = np.asarray(lengths, dtype=np.int64)
+    n0 = np.asarray(n0, dtype=np.int64)
+    pairs_tok = int((T[:, None] * mask).sum())
+    # sum over tokens t of (n0 + t + 1) = T n0 + T (T + 1) / 2
+    att_pos = (T * n0 + T * (T + 1) // 2)[:, None] * mask
+    flops = 2 * s.layer_params * pairs_tok + int(4 * s.n_q_heads * s.head_dim * att_pos.sum())
+    kv_row = s.kv_dim * s.elem_bytes
+    w_union = int(mask.any(axis=0).sum()) * layer_weight_bytes(s)
+    kv = int(2 * kv_row * ((T + n0)[:, None] * mask).sum())
+    hid = int(T.sum()) * s.d_model * 4 * 2
+    return {"flops": flops, "bytes": w_union + kv + hid, "tokens": int(T.sum()), "gemm_flops":
+            2 * s.layer_params * pairs_tok}
+
+
 def roofline_seconds(cost: dict, hbm_gbs: float, tflops: float) -> float:
     return max(cost["bytes"] / (hbm_gbs * 1e9), cost["flops"] / (tflops * 1e12))
