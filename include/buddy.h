@@ -309,7 +309,9 @@ BUDDY_API int buddy_set_options(buddy_ctx* ctx, int32_t use_graph);
 
 /* Which kernels a context runs (valid after buddy_set_weights), so that a
  * measurement can state them: paths[0] GEMM (0 CUDA-core fp32, 1 tcgen05
- * bf16), paths[1] attention (0 CUDA-core, 1 mma.sync tensor-core loop),
+ * bf16), paths[1] attention (0 CUDA-core, 1 mma.sync tensor-core loop over
+ * the whole GPU, 2 the same contractions with one thread-block cluster per
+ * (row, KV head) stream, for small batches),
  * paths[2] RMSNorm computed inside the QKV and gate/up GEMMs (0/1),
  * paths[3] split-K sums in a separate fixup kernel (0/1).  n <= 4 entries. */
 BUDDY_API int buddy_get_paths(buddy_ctx* ctx, int32_t* paths, int32_t n);

@@ -271,7 +271,8 @@ class Context:
         v = (c_i32 * 4)()
         _check(self.lib.buddy_get_paths(self.handle, v, 4), "buddy_get_paths")
         return {"gemm": "tcgen05 bf16 (TMA, TMEM)" if v[0] else "CUDA-core fp32",
-                "attention": "mma.sync tensor-core" if v[1] else "CUDA-core",
+                "attention": ["CUDA-core", "mma.sync tensor-core, span merge kernel",
+                              "mma.sync tensor-core, one cluster per stream (DSMEM merge)"][v[1]],
                 "rmsnorm": "inside the QKV and gate/up GEMMs" if v[2] else "separate kernel",
                 "split_k_fixup": "separate kernel" if v[3] else "last-arriving CTA"}
 

@@ -12,7 +12,7 @@ CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libbuddy.so")
 SOURCES = ["api.cu", "kernels.cu", "attention.cu", "gemm_simt.cu", "gemm_tc.cu", "noalloc.cu", "gemm_pf.cu",
-           "attn_pf.cu", "prefill.cu"]
+           "attn_pf.cu", "prefill.cu", "attn_cl.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
          "--expt-relaxed-constexpr", "-Xptxas", "-warn-spills"]

@@ -271,7 +271,8 @@ extern "C" int buddy_get_paths(buddy_ctx* ctx, int32_t* paths, int32_t n) {
   if (!ctx || !paths || n < 0 || n > 4) return BUDDY_ERR_ARG;
   const Ctx& c = ctx->c;
   if (!c.have_weights) return BUDDY_ERR_STATE;
-  const int32_t v[4] = {c.use_tc ? 1 : 0, attention_tc(c) ? 1 : 0, (c.use_tc && c.tc_panel) ? 1 : 0,
+  const int32_t v[4] = {c.use_tc ? 1 : 0, attention_cl(c) ? 2 : (attention_tc(c) ? 1 : 0),
+                        (c.use_tc && c.tc_panel) ? 1 : 0,
                         (c.use_tc && c.tc_defer) ? 1 : 0};
   for (int i = 0; i < n; ++i) paths[i] = v[i];
   return BUDDY_OK;
@@ -379,7 +380,7 @@ static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, c
     ProfScope p(c, s, BUDDY_PROF_ATTENTION, 1, prof);
     launch_attention(c, sel, kv, l, c.q, c.attn_out, split ? c.attn_lo : nullptr, s);
   }
-  if (attention_tc(c)) {
+  if (attention_tc(c) && !attention_cl(c)) {
     ProfScope p(c, s, BUDDY_PROF_ATTN_MERGE, 1, prof);
     launch_attention_merge(c, sel, c.attn_out, split ? c.attn_lo : nullptr, s);
   }

@@ -137,7 +137,9 @@ void launch_attention_merge(const Ctx& c, RowSel sel, void* out, void* out_lo, c
 
 void launch_attention(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q,
                       void* out, void* out_lo, cudaStream_t s) {
-  if (attention_tc(c)) {
+  if (attention_cl(c)) {
+    launch_attention_cl(c, sel, kv, layer, q, out, out_lo, s);
+  } else if (attention_tc(c)) {
     if (c.hd == 128) {
       if (out_lo) attn_tc_impl<128, true>(c, sel, kv, layer, q, out, out_lo, s);
       else attn_tc_impl<128, false>(c, sel, kv, layer, q, out, out_lo, s);

@@ -122,6 +122,9 @@ void launch_attention(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int la
                       void* attn_out, void* attn_lo, cudaStream_t s);   // attention.cu
 int attention_max_spans(int max_pos);   // span partials per (row, query head)
 bool attention_tc(const Ctx& c);         // tensor-core loop: launch_attention_merge follows
+bool attention_cl(const Ctx& c);         // small batches: one cluster per stream, no merge kernel (attn_cl.cu)
+void launch_attention_cl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q, void* out,
+                         void* out_lo, cudaStream_t s);
 void launch_attention_merge(const Ctx& c, RowSel sel, void* out, void* out_lo, cudaStream_t s);
 void launch_route(const Ctx& c, int B, const float* h1, const float* pool, const int32_t* len,
                   int len_bias, const int32_t* k, uint8_t* mask, int32_t* sel, float* scores,
