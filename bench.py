@@ -463,6 +463,20 @@ def run_ours(args, ws, rank, local):
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
     w = C.BY_NAME[args.workload]
+    if args.prefill_only:
+        # the routed prefill alone (a prefill workload): one JSON line
+        r = measure_prefill(w, args.steps, args.warmup, dev, ws, local)
+        out = {"metric": "routed prefill tokens/s at 1 GB300", "value": r["value"], "unit": "tokens/s",
+               "n_gpus": ws, "steps": args.steps, "warmup": args.warmup, "ms_per_step": r["ms_per_call"],
+               "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": w.shape.dtype,
+               "data": "synthetic (seeded counter-based generator)", "config": {"workload": w.name}}
+        out.update({k: v for k, v in r.items() if k not in ("value", "unit")})
+        if rank == 0:
+            print(json.dumps(out), flush=True)
+        if ws > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return
     head = measure(w, args.steps, args.warmup, dev, ws, local, use_graph=not args.no_graph)
     out = {"metric": METRIC, "value": head["value"], "unit": "tokens/s", "n_gpus": ws, "steps": args.steps,
            "warmup": args.warmup, "ms_per_step": head["ms_per_step"], "higher_is_better": True,
@@ -525,6 +539,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--headline-only", action="store_true", help="skip the per_config workloads")
+    ap.add_argument("--prefill-only", action="store_true",
+                    help="time the routed prefill of --workload (a prefill workload) alone")
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline oracle sample")
     args = ap.parse_args()

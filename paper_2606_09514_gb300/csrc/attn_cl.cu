@@ -7,16 +7,17 @@
 // streaming.  Here a cluster of C CTAs (C = 16 where the device allows it,
 // else 8) takes one stream: CTA r streams positions [r np / C, (r+1) np / C)
 // with its 4 warps (contiguous quarters, 32-position chunks through a
-// 3-buffer cp.async ring per warp; the contractions are those of the
+// 2-buffer cp.async ring per warp; the contractions are those of the
 // tensor-core loop in attn_tc.cuh: S^T = K Q^T and O^T += V^T P^T on
 // mma.sync m16n8k16 with the G <= 8 query heads as the 8 columns, base-2
-// online softmax).  The 4 warps' partials are merged in shared memory, the
-// cluster synchronises, and CTA 0 merges the C CTA partials read through
-// distributed shared memory (log-sum-exp, in rank order: deterministic) and
-// writes the output; a second cluster barrier keeps every CTA's shared
-// memory alive until then.  No kernel-wide or cross-cluster waits; every CTA
-// reaches both cluster barriers (a cluster whose row is past the row count
-// leaves before the first, all of its CTAs together).
+// online softmax).  The 4 warps' partials are merged in shared memory and
+// every CTA stores its partial into CTA 0's gather area through distributed
+// shared memory (st.shared::cluster); after one cluster barrier (release /
+// acquire) CTA 0 merges the C partials from its own shared memory
+// (log-sum-exp, in rank order: deterministic) and writes the output.  No
+// kernel-wide or cross-cluster waits; every CTA reaches the cluster barrier
+// (a cluster whose row is past the row count leaves before it, all of its
+// CTAs together).
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -30,7 +31,8 @@ namespace buddy {
 constexpr int kClWarps = 4;
 constexpr int kClThreads = 32 * kClWarps;
 constexpr int kClChunk = 32;
-constexpr int kClStages = 3;
+constexpr int kClStages = 2;
+constexpr int kClMaxCtas = 16;
 
 constexpr int kClMaxStreams = 64;   // (rows x KV heads) up to which the cluster kernel is used
 
@@ -41,10 +43,11 @@ __host__ __device__ constexpr size_t attn_cl_bufs() {
 }
 template <int HD>
 __host__ __device__ constexpr size_t attn_cl_smem() {
-  // the warps' partials and the CTA's (m, l per head, o per head and channel)
-  // reuse the buffers once the streaming is done
-  const size_t parts = (size_t)(kClWarps + 1) * 8 * (HD + 2) * 4;
-  return attn_cl_bufs<HD>() > parts ? attn_cl_bufs<HD>() : parts;
+  // the warps' partials (m, l per head, o per head and channel) reuse the
+  // buffers once the streaming is done; then CTA 0's gather area, one
+  // partial per CTA of the cluster
+  const size_t parts = (size_t)kClWarps * 8 * (HD + 2) * 4;
+  return (attn_cl_bufs<HD>() > parts ? attn_cl_bufs<HD>() : parts) + (size_t)kClMaxCtas * 8 * (HD + 2) * 4;
 }
 
 __device__ __forceinline__ uint32_t cluster_rank() {
@@ -68,10 +71,8 @@ __device__ __forceinline__ uint32_t dsmem_addr(const void* p, uint32_t rank) {
                : "r"((uint32_t)__cvta_generic_to_shared(p)), "r"(rank));
   return r;
 }
-__device__ __forceinline__ float ld_dsmem(uint32_t addr) {
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
-  return v;
+__device__ __forceinline__ void st_dsmem(uint32_t addr, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
 }
 
 template <int HD, bool SPLIT>
@@ -104,7 +105,8 @@ __global__ void __launch_bounds__(kClThreads) attn_cl_kernel(AttnArgs<bf16> A) {
   bf16* wbuf = reinterpret_cast<bf16*>(smraw) + (size_t)warp * NST * 2 * CH * KROW;
   float* parts = reinterpret_cast<float*>(smraw);   // overlays the buffers after the streaming
   float* mine = parts + (size_t)warp * PSTRIDE;
-  float* ctap = parts + (size_t)kClWarps * PSTRIDE;
+  constexpr size_t kBufBytes = attn_cl_smem<HD>() - (size_t)kClMaxCtas * 8 * (HD + 2) * 4;
+  float* gather = reinterpret_cast<float*>(smraw + kBufBytes);   // CTA 0: one partial per CTA
 
   auto issue = [&](int p, int cnt, int buf) {
     bf16* Kd = wbuf + (size_t)buf * 2 * CH * KROW;
@@ -290,7 +292,9 @@ __global__ void __launch_bounds__(kClThreads) attn_cl_kernel(AttnArgs<bf16> A) {
     }
   }
   __syncthreads();
-  // the CTA's partial: the warps' partials merged per (head, channel)
+  // the CTA's partial, the warps' partials merged per (head, channel), stored
+  // into CTA 0's gather area
+  float* dst = gather + (size_t)rank * PSTRIDE;
   for (int x = tid; x < G * HD; x += kClThreads) {
     const int hh = x / HD, ch = x - hh * HD;
     float M = -INFINITY;
@@ -304,30 +308,29 @@ __global__ void __launch_bounds__(kClThreads) attn_cl_kernel(AttnArgs<bf16> A) {
       L += f * parts[w * PSTRIDE + 8 + hh];
       Ov += f * parts[w * PSTRIDE + 16 + hh * HD + ch];
     }
-    ctap[16 + hh * HD + ch] = Ov;
+    st_dsmem(dsmem_addr(dst + 16 + hh * HD + ch, 0), Ov);
     if (ch == 0) {
-      ctap[hh] = M;
-      ctap[8 + hh] = L;
+      st_dsmem(dsmem_addr(dst + hh, 0), M);
+      st_dsmem(dsmem_addr(dst + 8 + hh, 0), L);
     }
   }
-  cluster_sync();   // every CTA's partial is written and visible to the cluster
+  cluster_sync();   // every CTA's partial has landed in CTA 0's gather area
   if (rank == 0) {
     const size_t obase = ((size_t)j * nq + (size_t)g * G) * HD;
     for (int x = tid; x < G * HD; x += kClThreads) {
       const int hh = x / HD, ch = x - hh * HD;
       float M = -INFINITY;
-      for (uint32_t r = 0; r < C; ++r) M = fmaxf(M, ld_dsmem(dsmem_addr(ctap + hh, r)));
+      for (uint32_t r = 0; r < C; ++r) M = fmaxf(M, gather[r * PSTRIDE + hh]);
       float L = 0.f, Ov = 0.f;
       for (uint32_t r = 0; r < C; ++r) {
-        const float mr = ld_dsmem(dsmem_addr(ctap + hh, r));
+        const float mr = gather[r * PSTRIDE + hh];
         const float f = mr == -INFINITY ? 0.f : tca::exp2a(mr - M);
-        L += f * ld_dsmem(dsmem_addr(ctap + 8 + hh, r));
-        Ov += f * ld_dsmem(dsmem_addr(ctap + 16 + hh * HD + ch, r));
+        L += f * gather[r * PSTRIDE + 8 + hh];
+        Ov += f * gather[r * PSTRIDE + 16 + hh * HD + ch];
       }
       store_out(A.out, A.out_lo, obase + (size_t)hh * HD + ch, Ov / L);
     }
   }
-  cluster_sync();   // CTA 0 has read every CTA's shared memory
 }
 
 // Cluster size the device schedules for this kernel: 16 CTAs where allowed,
@@ -339,7 +342,7 @@ static int cl_size(const Ctx& c) {
   const size_t smem = attn_cl_smem<HD>();
   cudaFuncSetAttribute(attn_cl_kernel<HD, SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   chosen = 0;
-  for (int C : {16, 8}) {
+  for (int C : {kClMaxCtas, 8}) {
     if (C > 8 && cudaFuncSetAttribute(attn_cl_kernel<HD, SPLIT>, cudaFuncAttributeNonPortableClusterSizeAllowed,
                                       1) != cudaSuccess) {
       cudaGetLastError();

@@ -219,6 +219,13 @@ PF_LLAMA3_B16 = Workload("llama3-8b-prefill-b16", LLAMA3_8B, batch=16, steps=1, 
                          description="Llama-3-8B shape, bf16, 16 prompts of U[128,1024] tokens, k=15 of 30")
 
 
+# Three-layer model with the same per-layer sizes, 4 prompts: kernel captures.
+P_PF_LLAMA3_3L_B4 = Workload("llama3-8b-3layer-prefill-b4",
+                             dataclasses.replace(LLAMA3_8B, name="llama3-8b-3layer", n_layers=3),
+                             batch=4, steps=1, seed=0, ctx_kind="fixed", ctx_args=(0,), k_kind="fixed",
+                             k_args=(1,))
+
+
 def prompt_lengths(w: Workload, lo: int = 128, hi: int = 1024) -> np.ndarray:
     """Seeded prompt lengths U[lo, hi] of a prefill workload."""
     rng = np.random.default_rng(np.random.SeedSequence([w.seed, 0x7066]))
@@ -250,7 +257,7 @@ T_VARIANTS = [
 ]
 
 BY_NAME = {w.name: w for w in FULL_WORKLOADS + [T_GQA, T_QWEN, T_F32, T_PRED, P_LLAMA3_3L_B1, P_QWEN_3L_B256,
-                                                PF_LLAMA3_B16] + T_VARIANTS}
+                                                PF_LLAMA3_B16, P_PF_LLAMA3_3L_B4] + T_VARIANTS}
 
 
 def with_shape(w: Workload, name: Optional[str] = None, **shape_changes) -> Workload:
