@@ -134,7 +134,7 @@ extern "C" int buddy_create(const buddy_config* cfg, buddy_ctx** out) {
       (e = dalloc(&c.attn_l, B * c.nq * c.attn_max_chunks)) ||
       (e = dalloc(&c.attn_acc, B * c.nq * c.attn_max_chunks * c.hd)) ||
       (e = dalloc(&c.attn_ctr, B * c.nkv)) || (e = dalloc(&c.attn_meta, B + 2)) ||
-      (e = dalloc(&c.dm_u, B * c.r)) || (e = dalloc(&c.mask, B * c.L)) ||
+      (e = dalloc(&c.dm_u, (size_t)kRouteZSlots * B * c.r)) || (e = dalloc(&c.mask, B * c.L)) ||
       (e = dalloc(&c.sel, B * c.Lm)) || (e = dalloc(&c.scores, B * c.Lm)) ||
       (e = dalloc(&c.rows, (size_t)c.L * B)) || (e = dalloc(&c.count, (size_t)c.L)) ||
       (e = dalloc(&c.h_in_stage, B * c.d)) || (e = dalloc(&c.h_out_stage, B * c.d)) ||
@@ -213,7 +213,7 @@ extern "C" int buddy_set_budget_predictor(buddy_ctx* ctx, const buddy_predictor_
   const int cols = c.r + (bp ? bp->hidden : 0);
   if (cols > c.dm_u_cols) {
     float* nu = nullptr;
-    CK(cudaMalloc(&nu, (size_t)c.maxB * cols * sizeof(float)));
+    CK(cudaMalloc(&nu, (size_t)kRouteZSlots * c.maxB * cols * sizeof(float)));
     cudaFree(c.dm_u);
     c.dm_u = nu;
     c.dm_u_cols = cols;

@@ -3,6 +3,8 @@
 // row compaction with zero K/V for skipped layers, and KV prefill.
 #include <cuda_runtime.h>
 
+#include <algorithm>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -275,12 +277,18 @@ void launch_pool_update(const Ctx& c, int B, const buddy_kv_state& kv, cudaStrea
 // ---------------------------------------------------------------------------
 // Router, part 1 (Sec. 4.3 + App. C.1 first linear layer):
 //   x_i = [ pool_sum[i] / (len[i] + len_bias), expanded over query heads ; h1[i] ]
-//   u[i][unit] = SiLU(b1[unit] + W1[unit] . x_i)
+//   z[i][unit] = W1[unit] . x_i       (bias and SiLU follow in part 2)
 // for the Decision Module's r hidden units and, after them, the Budget
-// Predictor's rp hidden units (same input, Sec. 4.4).  One warp per hidden
-// unit and up to 8 sequences; u has r + rp columns.
+// Predictor's rp hidden units (same input, Sec. 4.4); z has r + rp columns.
+// Small batches: one CTA per hidden unit and up to 8 sequences; its 8 warps
+// take 8 contiguous slices of the 2d-long dot product (four float4 loads of
+// W1 in flight per lane), then reduce through shared memory.  Larger batches
+// (route_hidden_tiled_kernel): a tiled fp32 GEMM whose K splits leave
+// partial sums that part 2 adds in split order.
 // ---------------------------------------------------------------------------
 constexpr int kRouteRows = 8;
+constexpr int kRouteTiledMin = 16;    // batches above this take the tiled router GEMM
+constexpr int kRtBM = 32, kRtBN = 64, kRtBK = 32;
 
 __global__ void __launch_bounds__(256) route_hidden_kernel(
     int B, int d, int hd, int group, int nkv, const float* __restrict__ h1,
@@ -290,10 +298,10 @@ __global__ void __launch_bounds__(256) route_hidden_kernel(
   pdl_wait();
   pdl_trigger();
   if (call_aborted(status)) return;
+  __shared__ float red[8][kRouteRows];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int unit = blockIdx.x * 8 + warp;
+  const int unit = blockIdx.x;
   const int i0 = blockIdx.y * kRouteRows;
-  if (unit >= r + rp) return;
   const int nr = min(kRouteRows, B - i0);
   float inv[kRouteRows];
 #pragma unroll
@@ -303,37 +311,115 @@ __global__ void __launch_bounds__(256) route_hidden_kernel(
   for (int t = 0; t < kRouteRows; ++t) acc[t] = 0.f;
   const float* wr = unit < r ? w1 + (size_t)unit * 2 * d : pw1 + (size_t)(unit - r) * 2 * d;
   const int kvd = nkv * hd;
-  // pooled part: x[k] = pool[(k / hd) / group * hd + k % hd] / n
-  for (int k = lane * 4; k < d; k += 128) {
+  const int per = ((2 * d + 7) / 8 + 3) & ~3;   // elements of a warp's slice (multiple of 4)
+  const int k0 = warp * per, k1 = min(2 * d, k0 + per);
+#pragma unroll 4
+  for (int k = k0 + lane * 4; k < k1; k += 128) {
     const float4 w = __ldg(reinterpret_cast<const float4*>(wr + k));
-    const int qh = k / hd, e = k - qh * hd;
-    const int pk = (qh / group) * hd + e;
+    if (k < d) {   // pooled half: x[k] = pool[(k / hd) / group * hd + k % hd] / n
+      const int qh = k / hd, e = k - qh * hd;
+      const int pk = (qh / group) * hd + e;
 #pragma unroll
-    for (int t = 0; t < kRouteRows; ++t) {
-      if (t < nr) {
-        const float4 pv = *reinterpret_cast<const float4*>(pool + (size_t)(i0 + t) * kvd + pk);
-        acc[t] += (w.x * pv.x + w.y * pv.y + w.z * pv.z + w.w * pv.w) * inv[t];
+      for (int t = 0; t < kRouteRows; ++t) {
+        if (t < nr) {
+          const float4 pv = *reinterpret_cast<const float4*>(pool + (size_t)(i0 + t) * kvd + pk);
+          acc[t] += (w.x * pv.x + w.y * pv.y + w.z * pv.z + w.w * pv.w) * inv[t];
+        }
       }
-    }
-  }
-  for (int k = lane * 4; k < d; k += 128) {
-    const float4 w = __ldg(reinterpret_cast<const float4*>(wr + d + k));
+    } else {
 #pragma unroll
-    for (int t = 0; t < kRouteRows; ++t) {
-      if (t < nr) {
-        const float4 hv = *reinterpret_cast<const float4*>(h1 + (size_t)(i0 + t) * d + k);
-        acc[t] += w.x * hv.x + w.y * hv.y + w.z * hv.z + w.w * hv.w;
+      for (int t = 0; t < kRouteRows; ++t) {
+        if (t < nr) {
+          const float4 hv = *reinterpret_cast<const float4*>(h1 + (size_t)(i0 + t) * d + (k - d));
+          acc[t] += w.x * hv.x + w.y * hv.y + w.z * hv.z + w.w * hv.w;
+        }
       }
     }
   }
 #pragma unroll
   for (int t = 0; t < kRouteRows; ++t) acc[t] = warp_sum(acc[t]);
-  if (lane < nr) {
+  if (lane == 0) {
+#pragma unroll
+    for (int t = 0; t < kRouteRows; ++t) red[warp][t] = acc[t];
+  }
+  __syncthreads();
+  if (threadIdx.x < nr) {
+    const int t = threadIdx.x;
     float v = 0.f;
 #pragma unroll
-    for (int t = 0; t < kRouteRows; ++t)
-      if (t == lane) v = acc[t];
-    u[(size_t)(i0 + lane) * (r + rp) + unit] = silu_f(v + (unit < r ? b1[unit] : pb1[unit - r]));
+    for (int w = 0; w < 8; ++w) v += red[w][t];
+    u[(size_t)(i0 + t) * (r + rp) + unit] = v;
+  }
+}
+
+// Router part 1 for larger batches: Z[i][unit] = X[i] . W[unit] over one K
+// split, tiles of 32 rows x 64 units, K in steps of 32 staged in shared
+// memory (transposed, so the inner loop reads consecutive addresses); each
+// of the 256 threads accumulates 2 rows x 4 units.  Split s writes its
+// partial sums to slot s of z ([splits, B, r + rp]).
+__global__ void __launch_bounds__(256) route_hidden_tiled_kernel(
+    int B, int d, int hd, int group, int nkv, const float* __restrict__ h1,
+    const float* __restrict__ pool, const int32_t* len, int len_bias, const float* __restrict__ w1, int r,
+    const float* __restrict__ pw1, int rp, int k_per_split, float* __restrict__ z, const int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
+  if (call_aborted(status)) return;
+  __shared__ float xs[kRtBK][kRtBM + 1];
+  __shared__ float ws[kRtBK][kRtBN + 1];
+  __shared__ float inv_s[kRtBM];
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  const int u0 = blockIdx.x * kRtBN, i0 = blockIdx.y * kRtBM;
+  const int cols = r + rp, kvd = nkv * hd;
+  const int ka = blockIdx.z * k_per_split, kb = min(2 * d, ka + k_per_split);
+  if (tid < kRtBM) inv_s[tid] = (i0 + tid < B) ? 1.0f / (float)(len[i0 + tid] + len_bias) : 0.f;
+  __syncthreads();
+  float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+  for (int k0 = ka; k0 < kb; k0 += kRtBK) {
+    // X tile: 32 rows x 32 columns (4 per thread)
+    for (int e = tid; e < kRtBM * kRtBK; e += 256) {
+      const int ri = e / kRtBK, kk = e - ri * kRtBK, k = k0 + kk, i = i0 + ri;
+      float v = 0.f;
+      if (i < B && k < kb) {
+        if (k < d) {
+          const int qh = k / hd, ee = k - qh * hd;
+          v = pool[(size_t)i * kvd + (qh / group) * hd + ee] * inv_s[ri];
+        } else {
+          v = h1[(size_t)i * d + (k - d)];
+        }
+      }
+      xs[kk][ri] = v;
+    }
+    // W tile: 64 units x 32 columns (8 per thread)
+    for (int e = tid; e < kRtBN * kRtBK; e += 256) {
+      const int ui = e / kRtBK, kk = e - ui * kRtBK, k = k0 + kk, unit = u0 + ui;
+      float v = 0.f;
+      if (unit < cols && k < kb)
+        v = unit < r ? __ldg(w1 + (size_t)unit * 2 * d + k) : __ldg(pw1 + (size_t)(unit - r) * 2 * d + k);
+      ws[kk][ui] = v;
+    }
+    __syncthreads();
+#pragma unroll 8
+    for (int kk = 0; kk < kRtBK; ++kk) {
+      const float a0 = xs[kk][ty * 2], a1 = xs[kk][ty * 2 + 1];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float b = ws[kk][tx * 4 + q];
+        acc[0][q] += a0 * b;
+        acc[1][q] += a1 * b;
+      }
+    }
+    __syncthreads();
+  }
+  float* zs = z + (size_t)blockIdx.z * B * cols;
+#pragma unroll
+  for (int a = 0; a < 2; ++a) {
+    const int i = i0 + ty * 2 + a;
+    if (i >= B) continue;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int unit = u0 + tx * 4 + q;
+      if (unit < cols) zs[(size_t)i * cols + unit] = acc[a][q];
+    }
   }
 }
 
@@ -343,22 +429,29 @@ __global__ void __launch_bounds__(256) route_hidden_kernel(
 // when s'[l'] > s'[l], or s'[l'] == s'[l] and l' < l.  A budget k_i = 0 takes
 // the Budget Predictor's k^ = 1 + argmax of its logits (ties to the smaller
 // k, Sec. 4.4).  Layers below `first` and the last layer are always set in
-// the mask.  One CTA per sequence; warps score layers (lanes split the dot
-// product).
-__global__ void __launch_bounds__(128) route_select_kernel(
-    int Lm, int first, int r, int rp, const float* __restrict__ u, const float* __restrict__ w2,
-    const float* __restrict__ b2, const float* __restrict__ prior, float omega,
-    const float* __restrict__ pw2, const float* __restrict__ pb2, const int32_t* k,
+// the mask.  One CTA per sequence; a warp per scored layer (and predictor
+// logit), its lanes splitting the dot product (eight loads in flight).
+__global__ void __launch_bounds__(1024) route_select_kernel(
+    int Lm, int first, int r, int rp, const float* __restrict__ z, int splits, int B, const float* __restrict__ b1,
+    const float* __restrict__ w2, const float* __restrict__ b2, const float* __restrict__ prior, float omega,
+    const float* __restrict__ pb1, const float* __restrict__ pw2, const float* __restrict__ pb2, const int32_t* k,
     uint8_t* mask, int32_t* sel, float* scores, const int32_t* status) {
   pdl_wait();
   pdl_trigger();
   if (call_aborted(status)) return;
   const int i = blockIdx.x;
-  extern __shared__ float s[];           // [Lm] scores, then [Lm] predictor logits
+  extern __shared__ float s[];           // [Lm] scores, [Lm] predictor logits, [r + rp] hidden units
   __shared__ int flag[kMaxLayers];
   __shared__ int kpred;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
-  const float* ui = u + (size_t)i * (r + rp);
+  float* ui = s + 2 * Lm;
+  // hidden units: K-split partial sums in split order, bias, SiLU
+  for (int c = threadIdx.x; c < r + rp; c += blockDim.x) {
+    float v = 0.f;
+    for (int sp = 0; sp < splits; ++sp) v += z[((size_t)sp * B + i) * (r + rp) + c];
+    ui[c] = silu_f(v + (c < r ? b1[c] : pb1[c - r]));
+  }
+  __syncthreads();
   const int ki0 = k[i];
   const bool predict = ki0 == 0 && pw2 != nullptr;
   for (int l = warp; l < (predict ? 2 * Lm : Lm); l += nw) {
@@ -368,7 +461,8 @@ __global__ void __launch_bounds__(128) route_select_kernel(
     const float* x = pl ? ui + r : ui;
     const int n = pl ? rp : r;
     float a = 0.f;
-    for (int t = lane; t < n; t += 32) a += w[t] * x[t];
+#pragma unroll 8
+    for (int t = lane; t < n; t += 32) a += __ldg(w + t) * x[t];
     a = warp_sum(a);
     if (lane == 0) {
       if (pl) {
@@ -413,16 +507,36 @@ __global__ void __launch_bounds__(128) route_select_kernel(
   if (threadIdx.x == 0 && mask) mask[(size_t)i * L + L - 1] = 1;
 }
 
+// K splits of the tiled router GEMM: about 128 CTAs, at most kRouteZSlots.
+static int route_splits(const Ctx& c, int B) {
+  if (B <= kRouteTiledMin) return 1;
+  const int cols = c.r + (c.have_pred ? c.pred.hidden : 0);
+  const int tiles = ((cols + kRtBN - 1) / kRtBN) * ((B + kRtBM - 1) / kRtBM);
+  return std::max(1, std::min(kRouteZSlots, 128 / std::max(1, tiles)));
+}
+
 void launch_route(const Ctx& c, int B, const float* h1, const float* pool, const int32_t* len,
                   int len_bias, const int32_t* k, uint8_t* mask, int32_t* sel, float* scores,
                   cudaStream_t s) {
   const int rp = c.have_pred ? c.pred.hidden : 0;
-  dim3 g1((c.r + rp + 7) / 8, (B + kRouteRows - 1) / kRouteRows);
-  launch_k(route_hidden_kernel, g1, 256, 0, s, c.pdl, B, c.d, c.hd, c.nq / c.nkv, c.nkv, h1, pool, len,
-           len_bias, c.dm.w1, c.dm.b1, c.r, c.have_pred ? c.pred.w1 : nullptr, c.have_pred ? c.pred.b1 : nullptr,
-           rp, c.dm_u, (const int32_t*)c.status);
-  launch_k(route_select_kernel, B, 128, 2 * c.Lm * sizeof(float), s, c.pdl, c.Lm, c.cl + 1, c.r, rp,
-           (const float*)c.dm_u, c.dm.w2, c.dm.b2, c.dm.prior, c.dm.omega, c.have_pred ? c.pred.w2 : nullptr,
+  const int cols = c.r + rp;
+  const int splits = route_splits(c, B);
+  if (B <= kRouteTiledMin) {
+    dim3 g1(cols, (B + kRouteRows - 1) / kRouteRows);
+    launch_k(route_hidden_kernel, g1, 256, 0, s, c.pdl, B, c.d, c.hd, c.nq / c.nkv, c.nkv, h1, pool, len,
+             len_bias, c.dm.w1, c.dm.b1, c.r, c.have_pred ? c.pred.w1 : nullptr, c.have_pred ? c.pred.b1 : nullptr,
+             rp, c.dm_u, (const int32_t*)c.status);
+  } else {
+    const int kps = ((2 * c.d + splits - 1) / splits + kRtBK - 1) / kRtBK * kRtBK;
+    dim3 g1((cols + kRtBN - 1) / kRtBN, (B + kRtBM - 1) / kRtBM, splits);
+    launch_k(route_hidden_tiled_kernel, g1, 256, 0, s, c.pdl, B, c.d, c.hd, c.nq / c.nkv, c.nkv, h1, pool, len,
+             len_bias, c.dm.w1, c.r, c.have_pred ? c.pred.w1 : nullptr, rp, kps, c.dm_u,
+             (const int32_t*)c.status);
+  }
+  const int sel_threads = 32 * std::min(32, (c.have_pred ? 2 : 1) * c.Lm);
+  launch_k(route_select_kernel, B, sel_threads, (2 * c.Lm + cols) * sizeof(float), s, c.pdl, c.Lm, c.cl + 1, c.r,
+           rp, (const float*)c.dm_u, splits, B, c.dm.b1, c.dm.w2, c.dm.b2, c.dm.prior, c.dm.omega,
+           c.have_pred ? c.pred.b1 : nullptr, c.have_pred ? c.pred.w2 : nullptr,
            c.have_pred ? c.pred.b2 : nullptr, k, mask, sel, scores, (const int32_t*)c.status);
 }
 

@@ -16,10 +16,11 @@ __global__ void route_hidden_kernel(int B, int d, int hd, int group, int nkv, co
                                     const float* pool, const int32_t* len, int len_bias,
                                     const float* w1, const float* b1, int r, const float* pw1,
                                     const float* pb1, int rp, float* u, const int32_t* status);
-__global__ void route_select_kernel(int Lm, int first, int r, int rp, const float* u, const float* w2,
-                                    const float* b2, const float* prior, float omega, const float* pw2,
-                                    const float* pb2, const int32_t* k, uint8_t* mask, int32_t* sel,
-                                    float* scores, const int32_t* status);
+__global__ void route_select_kernel(int Lm, int first, int r, int rp, const float* z, int splits, int B,
+                                    const float* b1, const float* w2, const float* b2, const float* prior,
+                                    float omega, const float* pb1, const float* pw2, const float* pb2,
+                                    const int32_t* k, uint8_t* mask, int32_t* sel, float* scores,
+                                    const int32_t* status);
 
 // Layout of the static scratch: words [0, 64) hold status (word 1 = abort
 // flag of the call in flight), then batch * dm_hidden fp32 hidden units.
@@ -94,12 +95,13 @@ extern "C" int buddy_route_noalloc(int32_t n_layers, int32_t d_model, int32_t n_
   cudaStream_t s = (cudaStream_t)stream;
   const int Lm = n_layers - 2;
   noalloc_check_kernel<<<1, 256, 0, s>>>(batch, k, Lm, len, status, flags_out);
-  dim3 g1((dm_hidden + 7) / 8, (batch + 7) / 8);
+  dim3 g1(dm_hidden, (batch + 7) / 8);
   route_hidden_kernel<<<g1, 256, 0, s>>>(batch, d_model, head_dim, n_q_heads / n_kv_heads, n_kv_heads,
                                          h1, pool_sum, len, 0, dm->w1, dm->b1, dm_hidden, nullptr, nullptr, 0,
                                          u, status);
-  route_select_kernel<<<batch, 128, 2 * Lm * sizeof(float), s>>>(Lm, 1, dm_hidden, 0, u, dm->w2, dm->b2,
-                                                                 dm->prior, dm->omega, nullptr, nullptr, k,
-                                                                 mask_out, sel_out, scores_out, status);
+  const int sel_threads = 32 * (Lm < 32 ? Lm : 32);
+  route_select_kernel<<<batch, sel_threads, (2 * Lm + dm_hidden) * sizeof(float), s>>>(
+      Lm, 1, dm_hidden, 0, u, 1, batch, dm->b1, dm->w2, dm->b2, dm->prior, dm->omega, nullptr, nullptr, nullptr, k,
+      mask_out, sel_out, scores_out, status);
   return cudaGetLastError() == cudaSuccess ? BUDDY_OK : BUDDY_ERR_CUDA;
 }
