@@ -53,7 +53,7 @@ static void free_ctx(buddy_ctx* x) {
   for (auto& kv : c.graphs) cudaGraphExecDestroy(kv.second);
   for (cudaEvent_t e : c.ev_pool) cudaEventDestroy(e);
   void* ptrs[] = {c.rope_cos, c.rope_sin, c.status, c.xn, c.act, c.attn_out, c.qkv, c.q,
-                  c.attn_m, c.attn_l, c.attn_acc, c.attn_ctr, c.dm_u, c.mask, c.sel, c.scores, c.rows,
+                  c.attn_m, c.attn_l, c.attn_acc, c.attn_ctr, c.dm_u, c.dm_x, c.mask, c.sel, c.scores, c.rows,
                   c.count, c.h_in_stage, c.h_out_stage, c.k_stage, c.mask_stage, c.xn_lo, c.act_lo, c.attn_lo,
                   c.gemm_ws, c.gemm_ctr, c.attn_meta, c.pf_xn, c.pf_xn_lo, c.pf_q, c.pf_attn, c.pf_attn_lo,
                   c.pf_act, c.pf_act_lo, c.pf_tok_seq, c.pf_tok_t, c.pf_tok_pos, c.pf_rows, c.pf_items,
@@ -134,7 +134,8 @@ extern "C" int buddy_create(const buddy_config* cfg, buddy_ctx** out) {
       (e = dalloc(&c.attn_l, B * c.nq * c.attn_max_chunks)) ||
       (e = dalloc(&c.attn_acc, B * c.nq * c.attn_max_chunks * c.hd)) ||
       (e = dalloc(&c.attn_ctr, B * c.nkv)) || (e = dalloc(&c.attn_meta, B + 2)) ||
-      (e = dalloc(&c.dm_u, (size_t)kRouteZSlots * B * c.r)) || (e = dalloc(&c.mask, B * c.L)) ||
+      (e = dalloc(&c.dm_u, (size_t)kRouteZSlots * B * c.r)) || (e = dalloc(&c.dm_x, B * 2 * c.d)) ||
+      (e = dalloc(&c.mask, B * c.L)) ||
       (e = dalloc(&c.sel, B * c.Lm)) || (e = dalloc(&c.scores, B * c.Lm)) ||
       (e = dalloc(&c.rows, (size_t)c.L * B)) || (e = dalloc(&c.count, (size_t)c.L)) ||
       (e = dalloc(&c.h_in_stage, B * c.d)) || (e = dalloc(&c.h_out_stage, B * c.d)) ||

@@ -14,7 +14,7 @@
 namespace buddy {
 
 constexpr int kMaxLayers = 128;
-constexpr int kRouteZSlots = 8;   // K-split slots of the router's hidden-unit partial sums
+constexpr int kRouteZSlots = 16;  // K-split slots of the router's hidden-unit partial sums
 constexpr int kMaxBatch = 1024;
 
 // Per-layer K/V base pointers passed by value to kernels that touch many layers.
@@ -197,6 +197,7 @@ struct Ctx {
   int32_t* attn_ctr = nullptr; // [maxB, nkv] chunk arrivals (self-resetting)
   int32_t* attn_meta = nullptr;   // [maxB + 2] row prefix and share (tensor-core attention)
   float* dm_u = nullptr;       // [kRouteZSlots, maxB, r + predictor hidden] partial sums
+  float* dm_x = nullptr;       // [maxB, 2d] router inputs (larger batches)
   uint8_t* mask = nullptr;     // [maxB, L]
   int32_t* sel = nullptr;      // [maxB, Lm]
   float* scores = nullptr;     // [maxB, Lm]

@@ -288,7 +288,7 @@ void launch_pool_update(const Ctx& c, int B, const buddy_kv_state& kv, cudaStrea
 // ---------------------------------------------------------------------------
 constexpr int kRouteRows = 8;
 constexpr int kRouteTiledMin = 16;    // batches above this take the tiled router GEMM
-constexpr int kRtBM = 32, kRtBN = 64, kRtBK = 32;
+constexpr int kRtBM = 64, kRtBN = 64, kRtBK = 32;
 
 __global__ void __launch_bounds__(256) route_hidden_kernel(
     int B, int d, int hd, int group, int nkv, const float* __restrict__ h1,
@@ -352,73 +352,105 @@ __global__ void __launch_bounds__(256) route_hidden_kernel(
   }
 }
 
-// Router part 1 for larger batches: Z[i][unit] = X[i] . W[unit] over one K
-// split, tiles of 32 rows x 64 units, K in steps of 32 staged in shared
-// memory (transposed, so the inner loop reads consecutive addresses); each
-// of the 256 threads accumulates 2 rows x 4 units.  Split s writes its
-// partial sums to slot s of z ([splits, B, r + rp]).
-__global__ void __launch_bounds__(256) route_hidden_tiled_kernel(
-    int B, int d, int hd, int group, int nkv, const float* __restrict__ h1,
-    const float* __restrict__ pool, const int32_t* len, int len_bias, const float* __restrict__ w1, int r,
-    const float* __restrict__ pw1, int rp, int k_per_split, float* __restrict__ z, const int32_t* status) {
+// Router part 1 for larger batches, step 1: the router input of every row,
+// X[i] = [pool_sum[i] / (len[i] + len_bias) expanded over query heads ; h1[i]]
+// ([B, 2d] fp32), so that the GEMM below reads plain rows.
+__global__ void __launch_bounds__(256) route_pack_kernel(int d, int hd, int group, int nkv,
+                                                         const float* __restrict__ h1,
+                                                         const float* __restrict__ pool, const int32_t* len,
+                                                         int len_bias, float* __restrict__ X,
+                                                         const int32_t* status) {
   pdl_wait();
   pdl_trigger();
   if (call_aborted(status)) return;
-  __shared__ float xs[kRtBK][kRtBM + 1];
-  __shared__ float ws[kRtBK][kRtBN + 1];
-  __shared__ float inv_s[kRtBM];
+  const int i = blockIdx.x;
+  const float inv = 1.0f / (float)(len[i] + len_bias);
+  const int kvd = nkv * hd;
+  float4* xo = reinterpret_cast<float4*>(X + (size_t)i * 2 * d);
+  for (int k = threadIdx.x * 4; k < 2 * d; k += blockDim.x * 4) {
+    float4 v;
+    if (k < d) {
+      const int qh = k / hd, e = k - qh * hd;
+      v = *reinterpret_cast<const float4*>(pool + (size_t)i * kvd + (qh / group) * hd + e);
+      v.x *= inv; v.y *= inv; v.z *= inv; v.w *= inv;
+    } else {
+      v = *reinterpret_cast<const float4*>(h1 + (size_t)i * d + (k - d));
+    }
+    xo[k >> 2] = v;
+  }
+}
+
+// Router part 1 for larger batches, step 2: Z[i][unit] = X[i] . W[unit] over
+// one K split.  Tiles of 64 rows x 64 units, K in steps of 32 staged in
+// shared memory (transposed: the inner loop reads 4 consecutive rows and 4
+// consecutive units as float4) with the next step's float4 loads in
+// registers while the current one is consumed; each of the 256 threads
+// accumulates 4 rows x 4 units.  Split s writes slot s of z ([splits, B,
+// r + rp]); part 2 adds the slots in split order.
+__global__ void __launch_bounds__(256) route_gemm_kernel(int B, int K2, const float* __restrict__ X,
+                                                         const float* __restrict__ w1, int r,
+                                                         const float* __restrict__ pw1, int rp, int k_per_split,
+                                                         float* __restrict__ z, const int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
+  if (call_aborted(status)) return;
+  __shared__ __align__(16) float xs[kRtBK][kRtBM + 4];
+  __shared__ __align__(16) float ws[kRtBK][kRtBN + 4];
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
   const int u0 = blockIdx.x * kRtBN, i0 = blockIdx.y * kRtBM;
-  const int cols = r + rp, kvd = nkv * hd;
-  const int ka = blockIdx.z * k_per_split, kb = min(2 * d, ka + k_per_split);
-  if (tid < kRtBM) inv_s[tid] = (i0 + tid < B) ? 1.0f / (float)(len[i0 + tid] + len_bias) : 0.f;
-  __syncthreads();
-  float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+  const int cols = r + rp;
+  const int ka = blockIdx.z * k_per_split, kb = min(K2, ka + k_per_split);
+  // this thread's two float4 of each tile: (row or unit) = e / 8, k4 = e % 8
+  float4 xr[2], wr[2];
+  auto fetch = [&](int k0) {
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const int e = tid + q * 256, rr = e >> 3, k = k0 + (e & 7) * 4;
+      const int i = i0 + rr, unit = u0 + rr;
+      xr[q] = (i < B && k < kb) ? *reinterpret_cast<const float4*>(X + (size_t)i * K2 + k)
+                                : make_float4(0.f, 0.f, 0.f, 0.f);
+      const float* wp = unit < r ? w1 + (size_t)unit * K2 : pw1 + (size_t)(unit - r) * K2;
+      wr[q] = (unit < cols && k < kb) ? __ldg(reinterpret_cast<const float4*>(wp + k))
+                                      : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  };
+  auto stash = [&]() {
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const int e = tid + q * 256, rr = e >> 3, kk = (e & 7) * 4;
+      xs[kk][rr] = xr[q].x; xs[kk + 1][rr] = xr[q].y; xs[kk + 2][rr] = xr[q].z; xs[kk + 3][rr] = xr[q].w;
+      ws[kk][rr] = wr[q].x; ws[kk + 1][rr] = wr[q].y; ws[kk + 2][rr] = wr[q].z; ws[kk + 3][rr] = wr[q].w;
+    }
+  };
+  float acc[4][4];
+#pragma unroll
+  for (int a = 0; a < 4; ++a) acc[a][0] = acc[a][1] = acc[a][2] = acc[a][3] = 0.f;
+  fetch(ka);
   for (int k0 = ka; k0 < kb; k0 += kRtBK) {
-    // X tile: 32 rows x 32 columns (4 per thread)
-    for (int e = tid; e < kRtBM * kRtBK; e += 256) {
-      const int ri = e / kRtBK, kk = e - ri * kRtBK, k = k0 + kk, i = i0 + ri;
-      float v = 0.f;
-      if (i < B && k < kb) {
-        if (k < d) {
-          const int qh = k / hd, ee = k - qh * hd;
-          v = pool[(size_t)i * kvd + (qh / group) * hd + ee] * inv_s[ri];
-        } else {
-          v = h1[(size_t)i * d + (k - d)];
-        }
-      }
-      xs[kk][ri] = v;
-    }
-    // W tile: 64 units x 32 columns (8 per thread)
-    for (int e = tid; e < kRtBN * kRtBK; e += 256) {
-      const int ui = e / kRtBK, kk = e - ui * kRtBK, k = k0 + kk, unit = u0 + ui;
-      float v = 0.f;
-      if (unit < cols && k < kb)
-        v = unit < r ? __ldg(w1 + (size_t)unit * 2 * d + k) : __ldg(pw1 + (size_t)(unit - r) * 2 * d + k);
-      ws[kk][ui] = v;
-    }
+    __syncthreads();   // the previous step's tiles are consumed
+    stash();
     __syncthreads();
+    if (k0 + kRtBK < kb) fetch(k0 + kRtBK);   // in flight while this step computes
 #pragma unroll 8
     for (int kk = 0; kk < kRtBK; ++kk) {
-      const float a0 = xs[kk][ty * 2], a1 = xs[kk][ty * 2 + 1];
+      const float4 a = *reinterpret_cast<const float4*>(&xs[kk][ty * 4]);
+      const float4 b = *reinterpret_cast<const float4*>(&ws[kk][tx * 4]);
+      const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float b = ws[kk][tx * 4 + q];
-        acc[0][q] += a0 * b;
-        acc[1][q] += a1 * b;
-      }
+      for (int p = 0; p < 4; ++p)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) acc[p][q] += av[p] * bv[q];
     }
-    __syncthreads();
   }
   float* zs = z + (size_t)blockIdx.z * B * cols;
 #pragma unroll
-  for (int a = 0; a < 2; ++a) {
-    const int i = i0 + ty * 2 + a;
+  for (int p = 0; p < 4; ++p) {
+    const int i = i0 + ty * 4 + p;
     if (i >= B) continue;
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const int unit = u0 + tx * 4 + q;
-      if (unit < cols) zs[(size_t)i * cols + unit] = acc[a][q];
+      if (unit < cols) zs[(size_t)i * cols + unit] = acc[p][q];
     }
   }
 }
@@ -507,12 +539,12 @@ __global__ void __launch_bounds__(1024) route_select_kernel(
   if (threadIdx.x == 0 && mask) mask[(size_t)i * L + L - 1] = 1;
 }
 
-// K splits of the tiled router GEMM: about 128 CTAs, at most kRouteZSlots.
+// K splits of the tiled router GEMM: about 256 CTAs, at most kRouteZSlots.
 static int route_splits(const Ctx& c, int B) {
   if (B <= kRouteTiledMin) return 1;
   const int cols = c.r + (c.have_pred ? c.pred.hidden : 0);
   const int tiles = ((cols + kRtBN - 1) / kRtBN) * ((B + kRtBM - 1) / kRtBM);
-  return std::max(1, std::min(kRouteZSlots, 128 / std::max(1, tiles)));
+  return std::max(1, std::min(kRouteZSlots, 256 / std::max(1, tiles)));
 }
 
 void launch_route(const Ctx& c, int B, const float* h1, const float* pool, const int32_t* len,
@@ -527,11 +559,12 @@ void launch_route(const Ctx& c, int B, const float* h1, const float* pool, const
              len_bias, c.dm.w1, c.dm.b1, c.r, c.have_pred ? c.pred.w1 : nullptr, c.have_pred ? c.pred.b1 : nullptr,
              rp, c.dm_u, (const int32_t*)c.status);
   } else {
+    launch_k(route_pack_kernel, B, 256, 0, s, c.pdl, c.d, c.hd, c.nq / c.nkv, c.nkv, h1, pool, len, len_bias,
+             c.dm_x, (const int32_t*)c.status);
     const int kps = ((2 * c.d + splits - 1) / splits + kRtBK - 1) / kRtBK * kRtBK;
     dim3 g1((cols + kRtBN - 1) / kRtBN, (B + kRtBM - 1) / kRtBM, splits);
-    launch_k(route_hidden_tiled_kernel, g1, 256, 0, s, c.pdl, B, c.d, c.hd, c.nq / c.nkv, c.nkv, h1, pool, len,
-             len_bias, c.dm.w1, c.r, c.have_pred ? c.pred.w1 : nullptr, rp, kps, c.dm_u,
-             (const int32_t*)c.status);
+    launch_k(route_gemm_kernel, g1, 256, 0, s, c.pdl, B, 2 * c.d, (const float*)c.dm_x, c.dm.w1, c.r,
+             c.have_pred ? c.pred.w1 : nullptr, rp, kps, c.dm_u, (const int32_t*)c.status);
   }
   const int sel_threads = 32 * std::min(32, (c.have_pred ? 2 : 1) * c.Lm);
   launch_k(route_select_kernel, B, sel_threads, (2 * c.Lm + cols) * sizeof(float), s, c.pdl, c.Lm, c.cl + 1, c.r,
