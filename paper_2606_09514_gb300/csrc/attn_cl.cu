@@ -12,12 +12,15 @@
 // mma.sync m16n8k16 with the G <= 8 query heads as the 8 columns, base-2
 // online softmax).  The 4 warps' partials are merged in shared memory and
 // every CTA stores its partial into CTA 0's gather area through distributed
-// shared memory (st.shared::cluster); after one cluster barrier (release /
-// acquire) CTA 0 merges the C partials from its own shared memory
-// (log-sum-exp, in rank order: deterministic) and writes the output.  No
-// kernel-wide or cross-cluster waits; every CTA reaches the cluster barrier
-// (a cluster whose row is past the row count leaves before it, all of its
-// CTAs together).
+// shared memory (st.shared::cluster), cut by output: the G x HD outputs of
+// the stream are split into C contiguous slices and CTA s owns slice s.
+// Every CTA stores its (m, l) of each head and its unnormalised output of
+// each (head, channel) into the gather area of that output's owner; after
+// one cluster barrier (release / acquire) every CTA merges the C partials of
+// its own slice from its own shared memory (log-sum-exp, in rank order:
+// deterministic) and writes those outputs.  No kernel-wide or cross-cluster
+// waits; every CTA reaches the cluster barrier (a cluster whose row is past
+// the row count leaves before it, all of its CTAs together).
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -41,13 +44,20 @@ __host__ __device__ constexpr size_t attn_cl_bufs() {
   // per warp: kClStages buffers of K and V rows (padded by 8 bf16)
   return (size_t)kClWarps * kClStages * 2 * kClChunk * (HD + 8) * 2;
 }
+// One partial in an owner's gather area: m[8], l[8], then the owner's slice
+// of outputs (at most 8 heads x HD channels / 8 CTAs).
+template <int HD>
+__host__ __device__ constexpr int attn_cl_gstride() {
+  return 16 + HD;
+}
 template <int HD>
 __host__ __device__ constexpr size_t attn_cl_smem() {
   // the warps' partials (m, l per head, o per head and channel) reuse the
-  // buffers once the streaming is done; then CTA 0's gather area, one
-  // partial per CTA of the cluster
+  // buffers once the streaming is done; then the gather area, one partial
+  // per CTA of the cluster
   const size_t parts = (size_t)kClWarps * 8 * (HD + 2) * 4;
-  return (attn_cl_bufs<HD>() > parts ? attn_cl_bufs<HD>() : parts) + (size_t)kClMaxCtas * 8 * (HD + 2) * 4;
+  return (attn_cl_bufs<HD>() > parts ? attn_cl_bufs<HD>() : parts) +
+         (size_t)kClMaxCtas * attn_cl_gstride<HD>() * 4;
 }
 
 __device__ __forceinline__ uint32_t cluster_rank() {
@@ -105,8 +115,9 @@ __global__ void __launch_bounds__(kClThreads) attn_cl_kernel(AttnArgs<bf16> A) {
   bf16* wbuf = reinterpret_cast<bf16*>(smraw) + (size_t)warp * NST * 2 * CH * KROW;
   float* parts = reinterpret_cast<float*>(smraw);   // overlays the buffers after the streaming
   float* mine = parts + (size_t)warp * PSTRIDE;
-  constexpr size_t kBufBytes = attn_cl_smem<HD>() - (size_t)kClMaxCtas * 8 * (HD + 2) * 4;
-  float* gather = reinterpret_cast<float*>(smraw + kBufBytes);   // CTA 0: one partial per CTA
+  constexpr int GS = attn_cl_gstride<HD>();
+  constexpr size_t kBufBytes = attn_cl_smem<HD>() - (size_t)kClMaxCtas * GS * 4;
+  float* gather = reinterpret_cast<float*>(smraw + kBufBytes);   // one partial per CTA of the cluster
 
   auto issue = [&](int p, int cnt, int buf) {
     bf16* Kd = wbuf + (size_t)buf * 2 * CH * KROW;
@@ -293,8 +304,8 @@ __global__ void __launch_bounds__(kClThreads) attn_cl_kernel(AttnArgs<bf16> A) {
   }
   __syncthreads();
   // the CTA's partial, the warps' partials merged per (head, channel), stored
-  // into CTA 0's gather area
-  float* dst = gather + (size_t)rank * PSTRIDE;
+  // into the gather area of the output's owner (slot `rank`)
+  const int SL = (G * HD + (int)C - 1) / (int)C;   // outputs per owner (<= HD for C >= 8)
   for (int x = tid; x < G * HD; x += kClThreads) {
     const int hh = x / HD, ch = x - hh * HD;
     float M = -INFINITY;
@@ -308,41 +319,47 @@ __global__ void __launch_bounds__(kClThreads) attn_cl_kernel(AttnArgs<bf16> A) {
       L += f * parts[w * PSTRIDE + 8 + hh];
       Ov += f * parts[w * PSTRIDE + 16 + hh * HD + ch];
     }
-    st_dsmem(dsmem_addr(dst + 16 + hh * HD + ch, 0), Ov);
+    const uint32_t own = (uint32_t)(x / SL);
+    float* slot = gather + (size_t)rank * GS;
+    st_dsmem(dsmem_addr(slot + 16 + (x - (int)own * SL), own), Ov);
+    // (m, l) of head hh to every owner whose slice holds one of its outputs
     if (ch == 0) {
-      st_dsmem(dsmem_addr(dst + hh, 0), M);
-      st_dsmem(dsmem_addr(dst + 8 + hh, 0), L);
+      const uint32_t o1 = (uint32_t)(((hh + 1) * HD - 1) / SL);
+      for (uint32_t o = own; o <= o1; ++o) {
+        st_dsmem(dsmem_addr(slot + hh, o), M);
+        st_dsmem(dsmem_addr(slot + 8 + hh, o), L);
+      }
     }
   }
-  cluster_sync();   // every CTA's partial has landed in CTA 0's gather area
-  if (rank == 0) {
-    const size_t obase = ((size_t)j * nq + (size_t)g * G) * HD;
-    for (int x = tid; x < G * HD; x += kClThreads) {
-      const int hh = x / HD, ch = x - hh * HD;
-      float M = -INFINITY;
-      for (uint32_t r = 0; r < C; ++r) M = fmaxf(M, gather[r * PSTRIDE + hh]);
-      float L = 0.f, Ov = 0.f;
-      for (uint32_t r = 0; r < C; ++r) {
-        const float mr = gather[r * PSTRIDE + hh];
-        const float f = mr == -INFINITY ? 0.f : tca::exp2a(mr - M);
-        L += f * gather[r * PSTRIDE + 8 + hh];
-        Ov += f * gather[r * PSTRIDE + 16 + hh * HD + ch];
-      }
-      store_out(A.out, A.out_lo, obase + (size_t)hh * HD + ch, Ov / L);
+  cluster_sync();   // every partial has landed in its owner's gather area
+  const size_t obase = ((size_t)j * nq + (size_t)g * G) * HD;
+  const int x0 = (int)rank * SL, x1 = min(G * HD, x0 + SL);
+  for (int x = x0 + tid; x < x1; x += kClThreads) {
+    const int hh = x / HD;
+    float M = -INFINITY;
+    for (uint32_t r = 0; r < C; ++r) M = fmaxf(M, gather[r * GS + hh]);
+    float L = 0.f, Ov = 0.f;
+    for (uint32_t r = 0; r < C; ++r) {
+      const float mr = gather[r * GS + hh];
+      const float f = mr == -INFINITY ? 0.f : tca::exp2a(mr - M);
+      L += f * gather[r * GS + 8 + hh];
+      Ov += f * gather[r * GS + 16 + (x - x0)];
     }
+    store_out(A.out, A.out_lo, obase + (size_t)x, Ov / L);
   }
 }
 
-// Cluster size the device schedules for this kernel: 16 CTAs where allowed,
-// else 8 (0 if neither).
+// Clusters of C CTAs the device can hold at once (C = 16 and 8), queried
+// once per instantiation; 0 where the size cannot be scheduled.
 template <int HD, bool SPLIT>
-static int cl_size(const Ctx& c) {
-  static int chosen = -1;   // one per instantiation
-  if (chosen >= 0) return chosen;
+static const int* cl_capacity() {
+  static int cap[2] = {-1, -1};   // [0]: C = 16, [1]: C = 8
+  if (cap[0] >= 0) return cap;
   const size_t smem = attn_cl_smem<HD>();
   cudaFuncSetAttribute(attn_cl_kernel<HD, SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  chosen = 0;
-  for (int C : {kClMaxCtas, 8}) {
+  for (int v = 0; v < 2; ++v) {
+    const int C = v == 0 ? kClMaxCtas : 8;
+    cap[v] = 0;
     if (C > 8 && cudaFuncSetAttribute(attn_cl_kernel<HD, SPLIT>, cudaFuncAttributeNonPortableClusterSizeAllowed,
                                       1) != cudaSuccess) {
       cudaGetLastError();
@@ -360,24 +377,31 @@ static int cl_size(const Ctx& c) {
     cfg.attrs = at;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, attn_cl_kernel<HD, SPLIT>, &cfg) == cudaSuccess && n > 0) {
-      chosen = C;
-      break;
-    }
+    if (cudaOccupancyMaxActiveClusters(&n, attn_cl_kernel<HD, SPLIT>, &cfg) == cudaSuccess) cap[v] = n;
     cudaGetLastError();
   }
-  return chosen;
+  return cap;
+}
+
+// Cluster size for `streams` streams: 16 CTAs when every cluster fits at
+// once (a cluster that waits for another to finish doubles the latency),
+// else 8; 0 if neither size can be scheduled.
+template <int HD, bool SPLIT>
+static int cl_size(int streams) {
+  const int* cap = cl_capacity<HD, SPLIT>();
+  if (cap[0] > 0 && (streams <= cap[0] || cap[1] <= 0)) return kClMaxCtas;
+  return cap[1] > 0 ? 8 : 0;
 }
 
 bool attention_cl(const Ctx& c) {
   if (!(c.dtype == BUDDY_DTYPE_BF16 && c.nq / c.nkv <= 8 && c.maxB * c.nkv <= kClMaxStreams)) return false;
-  return (c.hd == 128 ? cl_size<128, false>(c) : cl_size<64, false>(c)) > 0;
+  return (c.hd == 128 ? cl_size<128, false>(c.maxB * c.nkv) : cl_size<64, false>(c.maxB * c.nkv)) > 0;
 }
 
 template <int HD, bool SPLIT>
 static void attn_cl_impl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q, void* out,
                          void* out_lo, cudaStream_t s) {
-  const int C = cl_size<HD, SPLIT>(c);
+  const int C = cl_size<HD, SPLIT>(sel.n * c.nkv);
   AttnArgs<bf16> A{q, sel.rows, sel.count, sel.n, c.nq, c.nkv, cache_len(c, kv, layer), kv.seq_off, kv.cap,
                    (const bf16*)kv.k_cache[layer], (const bf16*)kv.v_cache[layer], 0, nullptr, nullptr, nullptr,
                    nullptr, (bf16*)out, (bf16*)out_lo, c.status, nullptr};

@@ -94,6 +94,7 @@ struct TcParams {
   uint32_t panel_off;     // byte offset of panel 0 in dynamic shared memory
   uint32_t panel_bytes;   // bytes of one panel (hi, then lo for SPLIT)
   int panel_kb;           // K blocks one panel holds (hi part)
+  uint32_t gstage_off;    // byte offset of the first unit's RMSNorm gains (fp32, panel_kb x 64)
   // Deferred fixup: units only stage their partials; a second kernel
   // (gemm_fix_kernel) sums the splits and applies the epilogue on every SM.
   int defer;
@@ -238,6 +239,65 @@ __device__ __forceinline__ void tc_panel_write(const TcParams& p, uint8_t* panel
         }
       }
       // row j of K block r: 16-byte chunk q / 2 of the row at chunk (q / 2) ^ j
+      const uint32_t off = (uint32_t)r * 1024u + (uint32_t)j * 128u + (uint32_t)((((q >> 1) ^ j) & 7) << 4) +
+                           (uint32_t)((q & 1) * 8);
+      *reinterpret_cast<uint2*>(panel + off) = make_uint2(hi[0], hi[1]);
+      if (SPLIT) *reinterpret_cast<uint2*>(panel + (size_t)p.panel_kb * 1024 + off) = make_uint2(lo[0], lo[1]);
+    }
+  }
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Largest K the single-pass first panel handles (one float4 per thread per
+// 512 columns, 16 per thread).
+constexpr int kPanelFirstMaxK = 16 * 512;
+
+// The first unit's panel in one pass over each row: every thread loads its
+// 16 float4 of row j (the loads of the sum of squares), the sum is reduced
+// across the 4 epilogue warps, and the thread then writes the panel entries
+// of the unit's K range [kb0, kb1) that it already holds, scaled by 1 / rms
+// and by the gains staged in shared memory (gst, from column kb0 * 64).  The
+// arithmetic (order of the squares, of the reduction and of the products) is
+// that of tc_panel_inv followed by tc_panel_write.  row_of[j] holds the
+// source row of panel row j.
+template <bool SPLIT>
+__device__ __forceinline__ void tc_panel_first(const TcParams& p, uint8_t* panel, int m, int kb0, int kb1, int et,
+                                               const int* row_of, const float* gst, float* red, float* inv) {
+  const int lane = et & 31, w = et >> 5;
+  const int c_lo = kb0 * kTileK, c_hi = kb1 * kTileK;
+  for (int j = 0; j < m; ++j) {
+    const float* h = p.nsrc + (size_t)row_of[j] * p.K;
+    float4 x[16];
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      const int e = (et + k * 128) * 4;
+      x[k] = e < p.K ? *reinterpret_cast<const float4*>(h + e) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    float ss = 0.f;
+#pragma unroll
+    for (int k = 0; k < 16; ++k) ss += x[k].x * x[k].x + x[k].y * x[k].y + x[k].z * x[k].z + x[k].w * x[k].w;
+    ss = warp_sum(ss);
+    if (lane == 0) red[j * 4 + w] = ss;
+    epi_bar();
+    const float iv = rsqrtf(((red[j * 4] + red[j * 4 + 1]) + (red[j * 4 + 2] + red[j * 4 + 3])) / (float)p.K + p.neps);
+    if (et == 0) inv[j] = iv;
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      const int e = (et + k * 128) * 4;
+      if (e < c_lo || e >= c_hi) continue;
+      const int c = e - c_lo, r = c >> 6, q = (c & 63) >> 2;
+      const float4 g = *reinterpret_cast<const float4*>(gst + c);
+      const float y[4] = {x[k].x * iv * g.x, x[k].y * iv * g.y, x[k].z * iv * g.z, x[k].w * iv * g.w};
+      uint32_t hi[2], lo[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const bf16 a = from_f<bf16>(y[2 * u]), c2 = from_f<bf16>(y[2 * u + 1]);
+        hi[u] = (uint32_t)__bfloat16_as_ushort(a) | ((uint32_t)__bfloat16_as_ushort(c2) << 16);
+        if (SPLIT) {
+          const bf16 la = from_f<bf16>(y[2 * u] - to_f(a)), lc = from_f<bf16>(y[2 * u + 1] - to_f(c2));
+          lo[u] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lc) << 16);
+        }
+      }
       const uint32_t off = (uint32_t)r * 1024u + (uint32_t)j * 128u + (uint32_t)((((q >> 1) ^ j) & 7) << 4) +
                            (uint32_t)((q & 1) * 8);
       *reinterpret_cast<uint2*>(panel + off) = make_uint2(hi[0], hi[1]);

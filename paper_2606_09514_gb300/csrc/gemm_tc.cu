@@ -42,6 +42,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __shared__ volatile int consumed;
   __shared__ int last_flag;
   __shared__ float pred[32], pinv[8];   // panel mode: sums of squares, 1 / rms per row
+  __shared__ int prow[8];               // panel mode: source row of each panel row
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -109,6 +110,21 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       }
     }
   }
+  const bool panel = p.nsrc != nullptr;
+  const bool first_pass = panel && p.K <= kPanelFirstMaxK;
+  if (first_pass && warp >= 2 && blockIdx.x < p.units) {
+    // Before the wait: the RMSNorm gains of the first unit's K range (weights,
+    // written by no kernel of the step) into shared memory, and the source
+    // rows (written by the compaction kernel, complete before this kernel
+    // could launch unless count_late, in which case the wait is behind us).
+    const int et = threadIdx.x - 64;
+    const int split = blockIdx.x / p.n_tiles;
+    const int kb0 = split * p.kb_per_split, kb1 = min(p.kb_total, kb0 + p.kb_per_split);
+    float* gst = reinterpret_cast<float*>(smem + p.gstage_off);
+    for (int c = et * 4; c < (kb1 - kb0) * kTileK; c += 128 * 4)
+      *reinterpret_cast<float4*>(gst + c) = *reinterpret_cast<const float4*>(p.ngamma + kb0 * kTileK + c);
+    if (et < 8 && et < p.n) prow[et] = p.rows ? p.rows[et] : et;
+  }
   if (!waited) pdl_wait();
   pdl_trigger();
   const int m = call_aborted(p.status) ? 0 : (p.count ? *p.count : p.n);
@@ -128,7 +144,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (warp == 1) ptx::tmem_dealloc(tmem_base, p.tmem_cols);
     return;
   }
-  const bool panel = p.nsrc != nullptr;
   const uint32_t x_bytes = panel ? 0u : tc_x_bytes(m, SPLIT);
   const uint32_t acc_cols = (uint32_t)(p.mt * p.bw);
 
@@ -230,11 +245,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     uint32_t acc_ph = 0;
     const int et = threadIdx.x - 64;
     if (panel && blockIdx.x < p.units) {
-      // the norm of every row, then the first unit's panel
-      tc_panel_inv(p, m, et, pred, pinv);
+      // the first unit's panel (and the norm of every row)
       const int split = blockIdx.x / p.n_tiles;
       const int kb0 = split * p.kb_per_split, kb1 = min(p.kb_total, kb0 + p.kb_per_split);
-      tc_panel_write<SPLIT>(p, smem + p.panel_off, m, kb0, kb1, et, pinv);
+      if (first_pass) {
+        epi_bar();   // staged gains and rows visible to all epilogue warps
+        tc_panel_first<SPLIT>(p, smem + p.panel_off, m, kb0, kb1, et, prow,
+                              reinterpret_cast<const float*>(smem + p.gstage_off), pred, pinv);
+      } else {
+        tc_panel_inv(p, m, et, pred, pinv);
+        tc_panel_write<SPLIT>(p, smem + p.panel_off, m, kb0, kb1, et, pinv);
+      }
       epi_bar();
       if (et == 0) ptx::mbar_arrive(&pfull_bar[0]);
     }
@@ -445,7 +466,8 @@ int gemm_tc_prepare(Ctx& c) {
   // Panel mode for up to eight rows: the QKV and gate/up GEMMs normalise their
   // own activations (no RMSNorm kernels, no activation copies).  Stages hold
   // weight tiles only; two panels of the largest K range follow the ring, then
-  // 15 KiB for the tail of an M = 128 operand read.
+  // 15 KiB for the tail of an M = 128 operand read, then the first unit's
+  // RMSNorm gains (staged before the dependency wait).
   c.tc_panel = c.maxB <= 8 && c.d % kTileK == 0;
   if (c.tc_panel) {
     int N, K, tiles;
@@ -456,7 +478,8 @@ int gemm_tc_prepare(Ctx& c) {
     const int limit = 227 * 1024 - 2 * 1024;
     for (int v = 0; v < 2; ++v) {
       c.tc_panel_bytes[v] = (uint32_t)(v + 1) * (uint32_t)c.tc_panel_kb * 1024u;
-      const int fixed = 1024 + 2 * (int)c.tc_panel_bytes[v] + 15 * 1024;
+      // + the first unit's RMSNorm gains (fp32)
+      const int fixed = 1024 + 2 * (int)c.tc_panel_bytes[v] + 15 * 1024 + c.tc_panel_kb * kTileK * 4;
       c.tc_pstages[v] = std::min(kTcMaxStages, (limit - fixed) / (c.tc_bw * 128));
       c.tc_psmem[v] = c.tc_pstages[v] * c.tc_bw * 128 + fixed;
       if (c.tc_pstages[v] < 3) c.tc_panel = false;
@@ -548,6 +571,7 @@ static TcParams tc_params(const Ctx& c, const GemmArgs& a, size_t* smem_out) {
     p.w_off = 0;
     p.panel_off = (uint32_t)p.stages * p.stage_bytes;
     p.panel_bytes = c.tc_panel_bytes[v];
+    p.gstage_off = p.panel_off + 2 * p.panel_bytes + 15 * 1024;
     p.panel_kb = c.tc_panel_kb;
     smem = c.tc_psmem[v];
   }
