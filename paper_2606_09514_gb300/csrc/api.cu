@@ -337,46 +337,69 @@ static void run_gemm(Ctx& c, int epi, GemmArgs a, int layer, int which, cudaStre
   }
 }
 
-// One decoder block on the rows of `sel` (Eq. 1 executed branch): the residual
-// stream H is updated in place for those rows; for layer 0 the input comes
-// from `src` and the output goes to `H`.
-static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, const float* src,
-                          float* H, cudaStream_t s, bool prof) {
+// GEMM arguments of one decoder block (Eq. 1 executed branch) on the rows of
+// `sel`: the residual stream H is updated in place for those rows; `src` is
+// the block's input (h_in for layer 0, else H).  Layers 0..c feed the router:
+// their GEMM inputs are kept as bf16 hi + lo pairs (split) so that the
+// routing input carries ~16 mantissa bits.  With `panel` the RMSNorms run
+// inside the QKV and gate/up GEMMs.
+static GemmArgs qkv_args(const Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, const float* src, bool split,
+                         bool panel) {
   const buddy_layer_weights& W = c.layers[l];
-  // Layers 0..c feed the router: their GEMM inputs are kept as bf16 hi + lo
-  // pairs so that the routing input carries ~16 mantissa bits.
-  const bool split = c.split0 && l <= c.cl;
-  const bool panel = c.use_tc && c.tc_panel;   // RMSNorms inside the QKV and gate/up GEMMs
-  if (!panel) {
-    ProfScope p(c, s, BUDDY_PROF_RMSNORM, 1, prof);
-    launch_rmsnorm(c, src, sel, W.attn_norm, c.xn, split ? c.xn_lo : nullptr, s);
-  }
   GemmArgs g{};
   g.sel = sel;
   g.max_m = sel.n;
   g.split = split;
   g.W = W.w_qkv; g.X = c.xn; g.X_lo = c.xn_lo; g.N = c.qkvN; g.K = c.d; g.out_f32 = c.qkv;
-  // the value-state feature is pooled in the QKV epilogue of the context
-  // layer; the other features by launch_pool_update
-  float* pool = (l == c.cl && c.feature == BUDDY_FEATURE_V) ? kv.pool_sum : nullptr;
   if (panel) {
     g.in_norm_src = src;
     g.in_norm_gamma = W.attn_norm;
-    // no RMSNorm kernel in between: the first middle layer's QKV GEMM follows
-    // the compaction kernel that writes its row count
-    g.count_late = l == c.cl + 1;
   }
+  // the value-state feature is pooled with the QKV finalisation of the
+  // context layer, the other features by launch_pool_update
+  g.pool = (l == c.cl && c.feature == BUDDY_FEATURE_V) ? kv.pool_sum : nullptr;
   if (c.use_tc) {
     // bias, RoPE, q, cache append and pool update in the GEMM epilogue
     g.qkv_bias = W.b_qkv; g.kv_len = kv.len; g.kv_seq_off = kv.seq_off; g.kv_cap = kv.cap;
     g.cache_len = cache_len(c, kv, l);
-    g.kc = kv.k_cache[l]; g.vc = kv.v_cache[l]; g.q_out = c.q; g.pool = pool;
-    run_gemm(c, EPI_QKV, g, l, 0, s, BUDDY_PROF_GEMM_QKV, prof);
-  } else {
-    run_gemm(c, EPI_STORE_F32, g, l, 0, s, BUDDY_PROF_GEMM_QKV, prof);
-    ProfScope p(c, s, BUDDY_PROF_QKV_FINALIZE, 1, prof);
-    launch_qkv_finalize(c, c.qkv, W.b_qkv, sel, kv, l, c.q, pool, s);
+    g.kc = kv.k_cache[l]; g.vc = kv.v_cache[l]; g.q_out = c.q;
   }
+  g.status = c.status;
+  g.layer = l;
+  g.which = 0;
+  return g;
+}
+static GemmArgs o_args(const Ctx& c, int l, RowSel sel, const float* src, float* H, bool split) {
+  GemmArgs g{};
+  g.sel = sel; g.max_m = sel.n; g.split = split;
+  g.W = c.layers[l].w_o; g.X = c.attn_out; g.X_lo = c.attn_lo; g.N = c.d; g.K = c.qd;
+  g.resid_src = src; g.resid_dst = H;
+  g.status = c.status; g.layer = l; g.which = 1;
+  return g;
+}
+static GemmArgs gate_up_args(const Ctx& c, int l, RowSel sel, float* H, bool split, bool panel) {
+  GemmArgs g{};
+  g.sel = sel; g.max_m = sel.n; g.split = split;
+  g.W = c.layers[l].w_gate_up; g.X = c.xn; g.X_lo = c.xn_lo; g.N = c.F; g.K = c.d; g.out_act = c.act;
+  if (panel) {
+    g.in_norm_src = H;
+    g.in_norm_gamma = c.layers[l].ffn_norm;
+  }
+  g.out_act_lo = split ? c.act_lo : nullptr;
+  g.status = c.status; g.layer = l; g.which = 2;
+  return g;
+}
+static GemmArgs down_args(const Ctx& c, int l, RowSel sel, float* H, bool split) {
+  GemmArgs g{};
+  g.sel = sel; g.max_m = sel.n; g.split = split;
+  g.W = c.layers[l].w_down; g.X = c.act; g.X_lo = c.act_lo; g.N = c.d; g.K = c.F;
+  g.resid_src = H; g.resid_dst = H;
+  g.status = c.status; g.layer = l; g.which = 3;
+  return g;
+}
+
+static void enqueue_attention(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, bool split, cudaStream_t s,
+                              bool prof) {
   {
     ProfScope p(c, s, BUDDY_PROF_ATTENTION, 1, prof);
     launch_attention(c, sel, kv, l, c.q, c.attn_out, split ? c.attn_lo : nullptr, s);
@@ -385,27 +408,37 @@ static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, c
     ProfScope p(c, s, BUDDY_PROF_ATTN_MERGE, 1, prof);
     launch_attention_merge(c, sel, c.attn_out, split ? c.attn_lo : nullptr, s);
   }
-  g = GemmArgs{};
-  g.sel = sel; g.max_m = sel.n; g.split = split;
-  g.W = W.w_o; g.X = c.attn_out; g.X_lo = c.attn_lo; g.N = c.d; g.K = c.qd; g.resid_src = src; g.resid_dst = H;
-  run_gemm(c, EPI_RESID, g, l, 1, s, BUDDY_PROF_GEMM_O, prof);
+}
+
+// One decoder block, one launch per GEMM.
+static void enqueue_layer(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, const float* src,
+                          float* H, cudaStream_t s, bool prof) {
+  const buddy_layer_weights& W = c.layers[l];
+  const bool split = c.split0 && l <= c.cl;
+  const bool panel = c.use_tc && c.tc_panel;
+  if (!panel) {
+    ProfScope p(c, s, BUDDY_PROF_RMSNORM, 1, prof);
+    launch_rmsnorm(c, src, sel, W.attn_norm, c.xn, split ? c.xn_lo : nullptr, s);
+  }
+  GemmArgs g = qkv_args(c, kv, l, sel, src, split, panel);
+  // no RMSNorm kernel in between: the first middle layer's QKV GEMM follows
+  // the compaction kernel that writes its row count
+  g.count_late = panel && l == c.cl + 1;
+  if (c.use_tc) {
+    run_gemm(c, EPI_QKV, g, l, 0, s, BUDDY_PROF_GEMM_QKV, prof);
+  } else {
+    run_gemm(c, EPI_STORE_F32, g, l, 0, s, BUDDY_PROF_GEMM_QKV, prof);
+    ProfScope p(c, s, BUDDY_PROF_QKV_FINALIZE, 1, prof);
+    launch_qkv_finalize(c, c.qkv, W.b_qkv, sel, kv, l, c.q, g.pool, s);
+  }
+  enqueue_attention(c, kv, l, sel, split, s, prof);
+  run_gemm(c, EPI_RESID, o_args(c, l, sel, src, H, split), l, 1, s, BUDDY_PROF_GEMM_O, prof);
   if (!panel) {
     ProfScope p(c, s, BUDDY_PROF_RMSNORM, 1, prof);
     launch_rmsnorm(c, H, sel, W.ffn_norm, c.xn, split ? c.xn_lo : nullptr, s);
   }
-  g = GemmArgs{};
-  g.sel = sel; g.max_m = sel.n; g.split = split;
-  g.W = W.w_gate_up; g.X = c.xn; g.X_lo = c.xn_lo; g.N = c.F; g.K = c.d; g.out_act = c.act;
-  if (panel) {
-    g.in_norm_src = H;
-    g.in_norm_gamma = W.ffn_norm;
-  }
-  g.out_act_lo = split ? c.act_lo : nullptr;
-  run_gemm(c, EPI_SWIGLU, g, l, 2, s, BUDDY_PROF_GEMM_GATE_UP, prof);
-  g = GemmArgs{};
-  g.sel = sel; g.max_m = sel.n; g.split = split;
-  g.W = W.w_down; g.X = c.act; g.X_lo = c.act_lo; g.N = c.d; g.K = c.F; g.resid_src = H; g.resid_dst = H;
-  run_gemm(c, EPI_RESID, g, l, 3, s, BUDDY_PROF_GEMM_DOWN, prof);
+  run_gemm(c, EPI_SWIGLU, gate_up_args(c, l, sel, H, split, panel), l, 2, s, BUDDY_PROF_GEMM_GATE_UP, prof);
+  run_gemm(c, EPI_RESID, down_args(c, l, sel, H, split), l, 3, s, BUDDY_PROF_GEMM_DOWN, prof);
 }
 
 struct StepIO {

@@ -138,18 +138,42 @@ __global__ void __launch_bounds__(kClThreads) attn_cl_kernel(AttnArgs<bf16> A) {
     }
   };
 
-  // prologue: chunks without the new token (position np - 1, written by the
-  // preceding kernel) may be copied before the wait
-  int xi = w0, k0 = 0;
-  for (; k0 < NST - 1 && xi < w1; ++k0) {
+  // prologue: every cached position may be copied before the wait; only the
+  // new token (position np - 1, written by the preceding kernel) comes after
+  // it, into the last row of its chunk.  A warp whose whole range fits in its
+  // NST buffers loads all of it here (the loop below then issues nothing);
+  // otherwise the first NST - 1 chunks, one buffer staying free for the loop.
+  const int pre = (w1 - w0 + CH - 1) / CH <= NST ? NST : NST - 1;
+  int xi = w0, k0 = 0, late_row = -1, late_buf = 0;
+  for (; k0 < pre && xi < w1; ++k0) {
     const int cnt = min(CH, w1 - xi);
-    if (xi + cnt == np) break;
+    if (xi + cnt == np) {
+      issue(xi, cnt - 1, k0);   // also zero-fills V rows cnt - 1 .. CH - 1
+      cp_async_commit();
+      late_row = cnt - 1;
+      late_buf = k0;
+      xi += cnt;
+      ++k0;
+      break;
+    }
     issue(xi, cnt, k0);
     cp_async_commit();
     xi += cnt;
   }
   pdl_wait();
   pdl_trigger();
+  if (late_row >= 0) {
+    __syncwarp();   // the zero fill of that row is done before the copy lands there
+    bf16* Kd = wbuf + (size_t)late_buf * 2 * CH * KROW + (size_t)late_row * KROW;
+    bf16* Vd = Kd + CH * KROW;
+    const bf16* ks = A.Kc + kvo + (int64_t)(np - 1) * HD;
+    const bf16* vs = A.Vc + kvo + (int64_t)(np - 1) * HD;
+    for (int x = lane; x < V16; x += 32) {
+      cp_async16(Kd + x * 8, ks + x * 8);
+      cp_async16(Vd + x * 8, vs + x * 8);
+    }
+    cp_async_commit();
+  }
   for (int k = k0; k < NST - 1; ++k) {
     if (xi < w1) {
       const int cnt = min(CH, w1 - xi);
