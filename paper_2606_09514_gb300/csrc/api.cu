@@ -327,7 +327,8 @@ static void run_gemm(Ctx& c, int epi, GemmArgs a, int layer, int which, cudaStre
       ProfScope p(c, s, cls, 1, prof);
       launch_gemm_tc(c, epi, a, s);
     }
-    if (c.tc_defer) {
+    // (a SwiGLU GEMM with one K split applies its epilogue itself)
+    if (c.tc_defer && !(epi == EPI_SWIGLU && c.tc_splits[which] == 1)) {
       ProfScope p(c, s, BUDDY_PROF_GEMM_FIXUP, 1, prof);
       launch_gemm_fix(c, epi, a, s);
     }

@@ -483,7 +483,9 @@ __device__ __forceinline__ void tc_fix_item(const TcParams& p, int tile, int j, 
 // (tempty) right after.  The CTA that completes a tile (the last of its K
 // splits, or the only one) then applies the epilogue with all 128 threads over
 // (row, 4-column group) items, summing the splits' slots in split order
-// (deterministic).  With p.defer every unit stops after staging its slot.
+// (deterministic).  With p.defer every unit stops after staging its slot,
+// except a SwiGLU GEMM with a single K split, which applies its epilogue
+// directly.
 // ---------------------------------------------------------------------------
 template <int EPI, bool SPLIT>
 __device__ __forceinline__ void tc_epilogue_unit(const TcParams& p, int u, int m, uint32_t tacc, uint64_t* tempty,
@@ -491,6 +493,54 @@ __device__ __forceinline__ void tc_epilogue_unit(const TcParams& p, int u, int m
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int q = warp & 3;   // TMEM lane quarter this warp may access
   const int tile = u % p.n_tiles;
+  if (EPI == EPI_SWIGLU && p.defer && p.splits == 1) {
+    // One K split (larger batches): SwiGLU straight from the accumulator, gate
+    // column c and up column c + bw/2 of the same row, with no workspace and no
+    // fixup kernel (the same arithmetic as tc_apply4 on a single partial).
+    const int h = p.bw >> 1;
+    for (int t = 0; t < p.mt; ++t) {
+      if (t * 128 + q * 32 >= m) continue;   // warp-uniform
+      const int j = t * 128 + q * 32 + lane;
+      const uint32_t ta = tacc + ((uint32_t)(q * 32) << 16) + (uint32_t)(t * p.bw);
+      for (int c0 = 0; c0 < h; c0 += 16) {
+        float g[16], up[16];
+        ptx::tmem_ld16(ta + c0, g);
+        ptx::tmem_ld16(ta + h + c0, up);
+        if (j >= m) continue;
+        const int f0 = tile * h + c0;
+        uint32_t hi[8], lo[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const float a0 = silu_f(g[2 * i]) * up[2 * i], a1 = silu_f(g[2 * i + 1]) * up[2 * i + 1];
+          const bf16 b0 = from_f<bf16>(a0), b1 = from_f<bf16>(a1);
+          hi[i] = (uint32_t)__bfloat16_as_ushort(b0) | ((uint32_t)__bfloat16_as_ushort(b1) << 16);
+          if (SPLIT) {
+            const bf16 l0 = from_f<bf16>(a0 - to_f(b0)), l1 = from_f<bf16>(a1 - to_f(b1));
+            lo[i] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+          }
+        }
+        bf16* dst = p.out_act + (size_t)j * p.N + f0;
+        bf16* dlo = SPLIT ? p.out_act_lo + (size_t)j * p.N + f0 : nullptr;
+        if (f0 + 16 <= p.N) {   // 32 bytes, 16-byte aligned (N % 8 == 0)
+          reinterpret_cast<uint4*>(dst)[0] = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+          reinterpret_cast<uint4*>(dst)[1] = make_uint4(hi[4], hi[5], hi[6], hi[7]);
+          if (SPLIT) {
+            reinterpret_cast<uint4*>(dlo)[0] = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+            reinterpret_cast<uint4*>(dlo)[1] = make_uint4(lo[4], lo[5], lo[6], lo[7]);
+          }
+        } else {
+          for (int i = 0; i < 16 && f0 + i < p.N; ++i) {
+            const uint32_t w = hi[i >> 1] >> ((i & 1) * 16);
+            dst[i] = __ushort_as_bfloat16((unsigned short)(w & 0xFFFFu));
+            if (SPLIT) dlo[i] = __ushort_as_bfloat16((unsigned short)((lo[i >> 1] >> ((i & 1) * 16)) & 0xFFFFu));
+          }
+        }
+      }
+    }
+    ptx::tc_fence_before();
+    if (lane == 0) ptx::mbar_arrive(tempty);
+    return;
+  }
   float4* slot = reinterpret_cast<float4*>(p.ws + (size_t)u * p.rows_max * p.bw);
   for (int t = 0; t < p.mt; ++t) {
     if (t * 128 + q * 32 >= m) continue;   // warp-uniform
