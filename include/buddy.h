@@ -27,6 +27,10 @@
  *   - Pointers marked "device" are device pointers owned by the caller; the
  *     library never frees them.  Weight pointers are retained (not copied) by
  *     buddy_set_weights and must stay valid while the context is used.
+ *   - Weight matrices and norm gains, the K/V caches, the pooled sums and the
+ *     hidden-state buffers (h_in, h_out, prefill x, route h1) must be 16-byte
+ *     aligned (the kernels access them with 16-byte vectors and TMA); a
+ *     misaligned one is rejected with BUDDY_ERR_ARG.
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
  *     Calls are asynchronous on that stream unless stated otherwise.
  *   - Return value: BUDDY_OK or a BUDDY_ERR_* code.  On a host-detected error

@@ -177,6 +177,9 @@ extern "C" void buddy_destroy(buddy_ctx* ctx) {
   free_ctx(ctx);
 }
 
+// Device buffers the kernels read or write with 16-byte vector accesses.
+static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
 extern "C" int buddy_set_weights(buddy_ctx* ctx, const buddy_layer_weights* layers,
                                  const buddy_dm_weights* dm) {
   if (!ctx || !layers || !dm) return BUDDY_ERR_ARG;
@@ -185,6 +188,9 @@ extern "C" int buddy_set_weights(buddy_ctx* ctx, const buddy_layer_weights* laye
     const buddy_layer_weights& w = layers[l];
     if (!w.attn_norm || !w.w_qkv || !w.w_o || !w.ffn_norm || !w.w_gate_up || !w.w_down)
       return BUDDY_ERR_ARG;
+    const void* wp[] = {w.attn_norm, w.w_qkv, w.w_o, w.ffn_norm, w.w_gate_up, w.w_down};
+    for (const void* p : wp)
+      if (!aligned16(p)) return BUDDY_ERR_ARG;
     if (c.cfg.qkv_bias && !w.b_qkv) return BUDDY_ERR_ARG;
   }
   if (!dm->w1 || !dm->b1 || !dm->w2 || !dm->b2) return BUDDY_ERR_ARG;
@@ -245,8 +251,10 @@ static int check_kv(const Ctx& c, const buddy_kv_state* kv, int need_batch) {
     return BUDDY_ERR_ARG;
   if (c.masked && !kv->layer_len) return BUDDY_ERR_ARG;
   if (kv->batch < need_batch || kv->batch < 1) return BUDDY_ERR_ARG;
+  if (!aligned16(kv->pool_sum)) return BUDDY_ERR_ARG;
   for (int l = 0; l < c.L; ++l)
-    if (!kv->k_cache[l] || !kv->v_cache[l]) return BUDDY_ERR_ARG;
+    if (!kv->k_cache[l] || !kv->v_cache[l] || !aligned16(kv->k_cache[l]) || !aligned16(kv->v_cache[l]))
+      return BUDDY_ERR_ARG;
   return BUDDY_OK;
 }
 
@@ -559,6 +567,7 @@ extern "C" int buddy_decode_step(buddy_ctx* ctx, const buddy_kv_state* kv, int32
   Ctx& c = ctx->c;
   if (!c.have_weights) return BUDDY_ERR_STATE;
   if (batch < 1 || batch > c.maxB || !h_in || !k || !h_out || h_in == h_out) return BUDDY_ERR_ARG;
+  if (!aligned16(h_in) || !aligned16(h_out)) return BUDDY_ERR_ARG;
   int rc = check_kv(c, kv, batch);
   if (rc) return rc;
   StepIO io{batch, h_in, k, h_out, mask_out, rows_out, count_out, scores_out};
@@ -595,6 +604,7 @@ extern "C" int buddy_prefill(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t b
   if (!c.have_weights) return BUDDY_ERR_STATE;
   if (c.pf_max <= 0 || c.dtype != BUDDY_DTYPE_BF16) return BUDDY_ERR_STATE;
   if (batch < 1 || batch > c.maxB || !n_tok || !x || !k || !h_out || x == h_out) return BUDDY_ERR_ARG;
+  if (!aligned16(x) || !aligned16(h_out)) return BUDDY_ERR_ARG;
   int rc = check_kv(c, kv, batch);
   if (rc) return rc;
   int64_t T = 0;
@@ -612,7 +622,7 @@ extern "C" int buddy_route(buddy_ctx* ctx, const buddy_kv_state* kv, int32_t bat
   if (!ctx) return BUDDY_ERR_ARG;
   Ctx& c = ctx->c;
   if (!c.have_weights) return BUDDY_ERR_STATE;
-  if (batch < 1 || batch > c.maxB || !h1 || !k) return BUDDY_ERR_ARG;
+  if (batch < 1 || batch > c.maxB || !h1 || !k || !aligned16(h1)) return BUDDY_ERR_ARG;
   if (!kv || !kv->len || !kv->pool_sum || !kv->cap || kv->batch < batch) return BUDDY_ERR_ARG;
   cudaStream_t s = (cudaStream_t)stream;
   // positions: the cache already holds the newest token (len >= 1)

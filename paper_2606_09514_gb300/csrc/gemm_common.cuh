@@ -345,11 +345,34 @@ __device__ __forceinline__ int tc_group_col(const TcParams& p, int g) {
   return g * 4;
 }
 
+__device__ __forceinline__ uint2 pack4_bf16(const float* y) {
+  return make_uint2((uint32_t)__bfloat16_as_ushort(from_f<bf16>(y[0])) |
+                        ((uint32_t)__bfloat16_as_ushort(from_f<bf16>(y[1])) << 16),
+                    (uint32_t)__bfloat16_as_ushort(from_f<bf16>(y[2])) |
+                        ((uint32_t)__bfloat16_as_ushort(from_f<bf16>(y[3])) << 16));
+}
+
 template <int EPI, bool SPLIT>
 __device__ __forceinline__ void tc_apply4(const TcParams& p, int tile, int j, int c, const float* v, const float* vp,
                                           const float* rs) {
   if (EPI == EPI_SWIGLU) {
     const int f0 = tile * (p.bw >> 1) + c;
+    if (f0 + 4 <= p.N) {   // one 8-byte store (N % 8 == 0, c % 4 == 0)
+      uint32_t hi[2], lo[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const float a0 = silu_f(v[2 * u]) * vp[2 * u], a1 = silu_f(v[2 * u + 1]) * vp[2 * u + 1];
+        const bf16 b0 = from_f<bf16>(a0), b1 = from_f<bf16>(a1);
+        hi[u] = (uint32_t)__bfloat16_as_ushort(b0) | ((uint32_t)__bfloat16_as_ushort(b1) << 16);
+        if (SPLIT) {
+          const bf16 l0 = from_f<bf16>(a0 - to_f(b0)), l1 = from_f<bf16>(a1 - to_f(b1));
+          lo[u] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+        }
+      }
+      *reinterpret_cast<uint2*>(p.out_act + (size_t)j * p.N + f0) = make_uint2(hi[0], hi[1]);
+      if (SPLIT) *reinterpret_cast<uint2*>(p.out_act_lo + (size_t)j * p.N + f0) = make_uint2(lo[0], lo[1]);
+      return;
+    }
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const int f = f0 + i;
@@ -385,45 +408,47 @@ __device__ __forceinline__ void tc_apply4(const TcParams& p, int tile, int j, in
       }
       if (head < p.nq) {
         float* q = p.q_out + (size_t)j * p.nq * hd + n0;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          q[i] = lo[i];
-          q[half + i] = hi[i];
-        }
+        *reinterpret_cast<float4*>(q) = make_float4(lo[0], lo[1], lo[2], lo[3]);
+        *reinterpret_cast<float4*>(q + half) = make_float4(hi[0], hi[1], hi[2], hi[3]);
       } else {
         bf16* k = p.kc + kv_offset(p.seq_off, p.cap, seq, p.nkv, hd, head - p.nq, cpos) + e0;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          k[i] = from_f<bf16>(lo[i]);
-          k[half + i] = from_f<bf16>(hi[i]);
-        }
+        *reinterpret_cast<uint2*>(k) = pack4_bf16(lo);
+        *reinterpret_cast<uint2*>(k + half) = pack4_bf16(hi);
       }
     } else {
       const int g = head - p.nq - p.nkv;
       bf16* vv = p.vc + kv_offset(p.seq_off, p.cap, seq, p.nkv, hd, g, cpos) + e0;
       float* pl = p.pool ? p.pool + (size_t)seq * p.nkv * hd + g * hd + e0 : nullptr;
+      *reinterpret_cast<uint2*>(vv) = pack4_bf16(x);
+      *reinterpret_cast<uint2*>(vv + half) = pack4_bf16(xp);
+      if (pl) {
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const bf16 a = from_f<bf16>(x[i]), b = from_f<bf16>(xp[i]);
-        vv[i] = a;
-        vv[half + i] = b;
-        if (pl) {
-          pl[i] += to_f(a);
-          pl[half + i] += to_f(b);
+        for (int i = 0; i < 4; ++i) {
+          pl[i] += to_f(from_f<bf16>(x[i]));
+          pl[half + i] += to_f(from_f<bf16>(xp[i]));
         }
       }
     }
   } else {
     const int n0 = tile * p.bw + c;
+    float* dst;
+    float w[4];
     if (EPI == EPI_STORE_F32) {
+      dst = p.out_f32 + (size_t)j * p.N + n0;
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
-        if (n0 + i < p.N) p.out_f32[(size_t)j * p.N + n0 + i] = v[i];
+      for (int i = 0; i < 4; ++i) w[i] = v[i];
     } else {
       const int seq = p.rows ? p.rows[j] : j;
+      dst = p.resid_dst + (size_t)seq * p.N + n0;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) w[i] = rs[i] + v[i];
+    }
+    if (n0 + 4 <= p.N) {   // one 16-byte store (N % 4 == 0, c % 4 == 0)
+      *reinterpret_cast<float4*>(dst) = make_float4(w[0], w[1], w[2], w[3]);
+    } else {
 #pragma unroll
       for (int i = 0; i < 4; ++i)
-        if (n0 + i < p.N) p.resid_dst[(size_t)seq * p.N + n0 + i] = rs[i] + v[i];
+        if (n0 + i < p.N) dst[i] = w[i];
     }
   }
 }
@@ -450,9 +475,15 @@ __device__ __forceinline__ void tc_fix_item(const TcParams& p, int tile, int j, 
   if (EPI == EPI_RESID) {
     const int seq = p.rows ? p.rows[j] : j;
     const int n0 = tile * p.bw + c;
+    const float* src = p.resid_src + (size_t)seq * p.N + n0;
+    if (n0 + 4 <= p.N) {
+      const float4 r4 = *reinterpret_cast<const float4*>(src);
+      rs[0] = r4.x; rs[1] = r4.y; rs[2] = r4.z; rs[3] = r4.w;
+    } else {
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
-      if (n0 + i < p.N) rs[i] = p.resid_src[(size_t)seq * p.N + n0 + i];
+      for (int i = 0; i < 4; ++i)
+        if (n0 + i < p.N) rs[i] = src[i];
+    }
   }
   for (int s0 = 0; s0 < p.splits; s0 += 8) {
     float4 x[8], y[8];

@@ -117,6 +117,17 @@ __device__ __forceinline__ float block_sum_256(float v, float* red) {
 // ---------------------------------------------------------------------------
 // RMSNorm with row gather: xn[j] = act(H[rows[j]] * rsqrt(mean(H^2) + eps) * g)
 // ---------------------------------------------------------------------------
+// Four consecutive values of a row as one vector store.
+__device__ __forceinline__ void store4(float* p, const float* y) {
+  *reinterpret_cast<float4*>(p) = make_float4(y[0], y[1], y[2], y[3]);
+}
+__device__ __forceinline__ void store4(bf16* p, const float* y) {
+  const bf16 a = from_f<bf16>(y[0]), b = from_f<bf16>(y[1]), c = from_f<bf16>(y[2]), e = from_f<bf16>(y[3]);
+  *reinterpret_cast<uint2*>(p) =
+      make_uint2((uint32_t)__bfloat16_as_ushort(a) | ((uint32_t)__bfloat16_as_ushort(b) << 16),
+                 (uint32_t)__bfloat16_as_ushort(c) | ((uint32_t)__bfloat16_as_ushort(e) << 16));
+}
+
 template <typename T>
 __global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ H, int d,
                                                       const int32_t* rows, const int32_t* count, int n,
@@ -132,6 +143,36 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ 
   const int i = rows ? rows[j] : j;
   __shared__ float red[32];
   const float* h = H + (size_t)i * d;
+  T* o = xn + (size_t)j * d;
+  T* olo = xn_lo ? xn_lo + (size_t)j * d : nullptr;
+  constexpr int R = 8;   // float4 of the row per thread: rows up to 8192 stay in registers
+  if (d <= 256 * 4 * R) {
+    float4 x[R];
+    float ss = 0.f;
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const int e = (threadIdx.x + r * 256) * 4;
+      x[r] = e < d ? *reinterpret_cast<const float4*>(h + e) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) ss += x[r].x * x[r].x + x[r].y * x[r].y + x[r].z * x[r].z + x[r].w * x[r].w;
+    ss = block_sum_256(ss, red);
+    const float inv = rsqrtf(ss / (float)d + eps);
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const int e = (threadIdx.x + r * 256) * 4;
+      if (e >= d) break;
+      const float4 g = *reinterpret_cast<const float4*>(gamma + e);
+      const float y[4] = {x[r].x * inv * g.x, x[r].y * inv * g.y, x[r].z * inv * g.z, x[r].w * inv * g.w};
+      store4(o + e, y);
+      if (olo) {   // remainder term (split activations)
+        const float z[4] = {y[0] - to_f(from_f<T>(y[0])), y[1] - to_f(from_f<T>(y[1])),
+                            y[2] - to_f(from_f<T>(y[2])), y[3] - to_f(from_f<T>(y[3]))};
+        store4(olo + e, z);
+      }
+    }
+    return;
+  }
   float ss = 0.f;
   for (int e = threadIdx.x * 4; e < d; e += blockDim.x * 4) {
     const float4 v = *reinterpret_cast<const float4*>(h + e);
@@ -139,17 +180,15 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ 
   }
   ss = block_sum_256(ss, red);
   const float inv = rsqrtf(ss / (float)d + eps);
-  T* o = xn + (size_t)j * d;
-  T* olo = xn_lo ? xn_lo + (size_t)j * d : nullptr;
   for (int e = threadIdx.x * 4; e < d; e += blockDim.x * 4) {
     const float4 v = *reinterpret_cast<const float4*>(h + e);
     const float4 g = *reinterpret_cast<const float4*>(gamma + e);
     const float y[4] = {v.x * inv * g.x, v.y * inv * g.y, v.z * inv * g.z, v.w * inv * g.w};
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const T hi = from_f<T>(y[u]);
-      o[e + u] = hi;
-      if (olo) olo[e + u] = from_f<T>(y[u] - to_f(hi));   // remainder term (split activations)
+    store4(o + e, y);
+    if (olo) {
+      const float z[4] = {y[0] - to_f(from_f<T>(y[0])), y[1] - to_f(from_f<T>(y[1])),
+                          y[2] - to_f(from_f<T>(y[2])), y[3] - to_f(from_f<T>(y[3]))};
+      store4(olo + e, z);
     }
   }
 }

@@ -241,6 +241,35 @@ def test_device_checks_write_nothing():
     assert not torch.all(h_out == 7.0)
 
 
+def test_misaligned_buffers_rejected_on_host():
+    """Hidden-state buffers and caches are accessed with 16-byte vectors: a
+    pointer off by 4 bytes is rejected before any launch (nothing written)."""
+    import paper_2606_09514_gb300 as pkg
+    w = C.T_GQA
+    dw = D.build(w)
+    s = w.shape
+    B = w.batch
+    h_in = synth.workload_h_in(w, 0, "cuda")
+    flat = torch.full((B * s.d_model + 4,), 7.0, device="cuda")
+    h_off = flat[1:1 + B * s.d_model].view(B, s.d_model)   # data_ptr() % 16 == 4
+    assert h_off.data_ptr() % 16 == 4
+    len0 = dw.kv.len.clone()
+    with pytest.raises(pkg.binding.BuddyError) as e:
+        dw.ctx.buddy_decode_step(dw.kv, h_in, dw.k, h_off)
+    assert e.value.code == pkg.binding.BUDDY_ERR_ARG
+    in_off = torch.empty(B * s.d_model + 4, device="cuda")[1:1 + B * s.d_model].view(B, s.d_model)
+    in_off.copy_(h_in)
+    h_out = torch.empty(B, s.d_model, device="cuda")
+    with pytest.raises(pkg.binding.BuddyError) as e:
+        dw.ctx.buddy_decode_step(dw.kv, in_off, dw.k, h_out)
+    assert e.value.code == pkg.binding.BUDDY_ERR_ARG
+    torch.cuda.synchronize()
+    assert torch.all(flat == 7.0) and torch.equal(dw.kv.len, len0)
+    # the context stays usable
+    dw.ctx.buddy_decode_step(dw.kv, h_in, dw.k, h_out)
+    assert dw.ctx.buddy_device_status() == 0
+
+
 def test_gemm_wait_limit_runs_out_and_context_recovers():
     """With a wait limit far below the time a TMA stage takes, the GEMMs give
     up: the step reports BUDDY_DEV_TIMEOUT.  Restoring the limit, the same
