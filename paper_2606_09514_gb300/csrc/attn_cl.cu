@@ -84,6 +84,11 @@ __device__ __forceinline__ uint32_t dsmem_addr(const void* p, uint32_t rank) {
 __device__ __forceinline__ void st_dsmem(uint32_t addr, float v) {
   asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
 }
+__device__ __forceinline__ void st_dsmem4(uint32_t addr, const float* v) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(v[0]), "f"(v[1]), "f"(v[2]),
+               "f"(v[3])
+               : "memory");
+}
 
 template <int HD, bool SPLIT>
 __global__ void __launch_bounds__(kClThreads) attn_cl_kernel(AttnArgs<bf16> A) {
@@ -328,24 +333,30 @@ __global__ void __launch_bounds__(kClThreads) attn_cl_kernel(AttnArgs<bf16> A) {
   }
   __syncthreads();
   // the CTA's partial, the warps' partials merged per (head, channel), stored
-  // into the gather area of the output's owner (slot `rank`)
+  // into the gather area of the output's owner (slot `rank`), four channels
+  // per thread and per 16-byte store (a slice is a multiple of 4 outputs:
+  // G * HD is a multiple of 64 and C is 8 or 16)
   const int SL = (G * HD + (int)C - 1) / (int)C;   // outputs per owner (<= HD for C >= 8)
-  for (int x = tid; x < G * HD; x += kClThreads) {
+  for (int x = tid * 4; x < G * HD; x += kClThreads * 4) {
     const int hh = x / HD, ch = x - hh * HD;
     float M = -INFINITY;
 #pragma unroll
     for (int w = 0; w < kClWarps; ++w) M = fmaxf(M, parts[w * PSTRIDE + hh]);
-    float L = 0.f, Ov = 0.f;
+    float L = 0.f, Ov[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int w = 0; w < kClWarps; ++w) {
       const float mw = parts[w * PSTRIDE + hh];
       const float f = mw == -INFINITY ? 0.f : tca::exp2a(mw - M);
       L += f * parts[w * PSTRIDE + 8 + hh];
-      Ov += f * parts[w * PSTRIDE + 16 + hh * HD + ch];
+      const float4 pv = *reinterpret_cast<const float4*>(parts + w * PSTRIDE + 16 + hh * HD + ch);
+      Ov[0] += f * pv.x;
+      Ov[1] += f * pv.y;
+      Ov[2] += f * pv.z;
+      Ov[3] += f * pv.w;
     }
     const uint32_t own = (uint32_t)(x / SL);
     float* slot = gather + (size_t)rank * GS;
-    st_dsmem(dsmem_addr(slot + 16 + (x - (int)own * SL), own), Ov);
+    st_dsmem4(dsmem_addr(slot + 16 + (x - (int)own * SL), own), Ov);
     // (m, l) of head hh to every owner whose slice holds one of its outputs
     if (ch == 0) {
       const uint32_t o1 = (uint32_t)(((hh + 1) * HD - 1) / SL);
@@ -358,18 +369,23 @@ __global__ void __launch_bounds__(kClThreads) attn_cl_kernel(AttnArgs<bf16> A) {
   cluster_sync();   // every partial has landed in its owner's gather area
   const size_t obase = ((size_t)j * nq + (size_t)g * G) * HD;
   const int x0 = (int)rank * SL, x1 = min(G * HD, x0 + SL);
-  for (int x = x0 + tid; x < x1; x += kClThreads) {
+  for (int x = x0 + tid * 4; x < x1; x += kClThreads * 4) {
     const int hh = x / HD;
     float M = -INFINITY;
     for (uint32_t r = 0; r < C; ++r) M = fmaxf(M, gather[r * GS + hh]);
-    float L = 0.f, Ov = 0.f;
+    float L = 0.f, Ov[4] = {0.f, 0.f, 0.f, 0.f};
     for (uint32_t r = 0; r < C; ++r) {
       const float mr = gather[r * GS + hh];
       const float f = mr == -INFINITY ? 0.f : tca::exp2a(mr - M);
       L += f * gather[r * GS + 8 + hh];
-      Ov += f * gather[r * GS + 16 + (x - x0)];
+      const float4 gv = *reinterpret_cast<const float4*>(gather + r * GS + 16 + (x - x0));
+      Ov[0] += f * gv.x;
+      Ov[1] += f * gv.y;
+      Ov[2] += f * gv.z;
+      Ov[3] += f * gv.w;
     }
-    store_out(A.out, A.out_lo, obase + (size_t)x, Ov / L);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) store_out(A.out, A.out_lo, obase + (size_t)(x + e), Ov[e] / L);
   }
 }
 
