@@ -36,7 +36,7 @@ METRIC = "budget-routed decode tokens/s at 1 GB300 per budget; % of HBM/tensor r
 # ncu dram bytes (read + write) per launch of the dominant kernel, from the
 # committed ncu summary of the gate/up GEMM (3-layer model with the same layer
 # shapes as the 32-layer bench workload); absent for kernels not captured
-NCU_TRAFFIC_PER_LAUNCH = {("llama3-8b-b1", "gemm_gate_up"): 238051840}
+NCU_TRAFFIC_PER_LAUNCH = {("llama3-8b-b1", "gemm_gate_up"): 238031616}
 DEFAULT_WORKLOAD = "llama3-8b-b1"
 PER_CONFIG = ["llama3-8b-b64-mixed", "llama2-13b-b32", "qwen2.5-7b-b256"]
 PREFILL_WORKLOAD = "llama3-8b-prefill-b16"
