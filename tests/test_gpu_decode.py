@@ -105,6 +105,26 @@ def test_decode_parity_bf16(w):
     assert worst < 2e-2
 
 
+# Batch sizes at the mode boundaries of the bf16 path: up to 8 rows the QKV
+# and gate/up GEMMs normalise in-kernel panels and the last K split applies
+# the epilogue, above 8 a fixup kernel does; up to 16 rows the router's first
+# layer is one CTA per hidden unit, above it a packed tiled GEMM; above 128
+# rows the GEMMs take two M-tiles.
+@pytest.mark.parametrize("base,batch", [(C.T_QWEN, 8), (C.T_QWEN, 9), (C.T_QWEN, 16), (C.T_QWEN, 17),
+                                        (C.T_QWEN, 128), (C.T_QWEN, 129), (C.T_GQA, 8), (C.T_GQA, 17)],
+                         ids=lambda v: v.shape.name if hasattr(v, "shape") else str(v))
+def test_decode_parity_batch_boundaries(base, batch):
+    if base.ctx_kind == "list":   # the listed contexts and budgets, repeated to the batch
+        ctx = [base.ctx_args[i % len(base.ctx_args)] for i in range(batch)]
+        k = [base.k_args[i % len(base.k_args)] for i in range(batch)]
+        w = C.scaled(base, ctx=ctx, k=k, name=f"{base.name}-b{batch}")
+    else:
+        w = C.scaled(base, batch=batch, name=f"{base.name}-b{batch}")
+    assert w.batch == batch
+    worst, _ = run_parity(w, steps=2)
+    assert worst < 2e-2
+
+
 def test_decode_parity_prior_and_graph():
     run_parity(C.T_GQA, steps=2, use_graph=True, prior=True)
 
