@@ -37,6 +37,19 @@ METRIC = "budget-routed decode tokens/s at 1 GB300 per budget; % of HBM/tensor r
 # committed ncu summary of the gate/up GEMM (3-layer model with the same layer
 # shapes as the 32-layer bench workload); absent for kernels not captured
 NCU_TRAFFIC_PER_LAUNCH = {("llama3-8b-b1", "gemm_gate_up"): 238031616}
+# DRAM traffic per algorithmic byte where the capture was a smaller case of
+# the same kernel whose traffic grows with the bytes it processes: the
+# attention of the 3-layer Qwen2.5-7B B=256 model (1,200,036,736 bytes of
+# traffic for 1,192,611,840 algorithmic bytes per launch)
+NCU_TRAFFIC_RATIO = {("qwen2.5-7b-b256", "attention"): 1200036736 / 1192611840}
+
+
+def _ncu_traffic(workload, kernel, bytes_per_launch):
+    if (workload, kernel) in NCU_TRAFFIC_PER_LAUNCH:
+        return NCU_TRAFFIC_PER_LAUNCH[(workload, kernel)]
+    if (workload, kernel) in NCU_TRAFFIC_RATIO:
+        return int(round(NCU_TRAFFIC_RATIO[(workload, kernel)] * bytes_per_launch))
+    return None
 DEFAULT_WORKLOAD = "llama3-8b-b1"
 PER_CONFIG = ["llama3-8b-b64-mixed", "llama2-13b-b32", "qwen2.5-7b-b256"]
 PREFILL_WORKLOAD = "llama3-8b-prefill-b16"
@@ -331,7 +344,7 @@ def measure(w, K, W, dev, ws, local, use_graph=True, e2e=True):
         avg_s = prof[dom][0] / 1e3 / launches
         ach = bytes_per_launch / avg_s / 1e9
         roof = {"bound": "hbm", "kernel": dom, "achieved": round(ach, 1), "peak": hbm, "unit": "GB/s",
-                "frac": round(ach / hbm, 4), "traffic": NCU_TRAFFIC_PER_LAUNCH.get((w.name, dom)),
+                "frac": round(ach / hbm, 4), "traffic": _ncu_traffic(w.name, dom, bytes_per_launch),
                 "bytes_per_launch": int(bytes_per_launch), "avg_launch_us": round(avg_s * 1e6, 2),
                 "launches": launches, "peak_source": f"{peak_src} hbm_gbs",
                 "frac_of_nominal": round(ach / NOMINAL_HBM_GBS, 4)}
@@ -344,7 +357,7 @@ def measure(w, K, W, dev, ws, local, use_graph=True, e2e=True):
     # the timed steps launch every routed layer (a layer no row selected exits
     # at once); the profiled steps launch only the selected ones
     per_layer = ("rmsnorm", "gemm_qkv", "qkv_finalize", "attention", "gemm_o", "gemm_gate_up", "gemm_down",
-                 "gemm_fixup", "attn_merge")
+                 "gemm_fixup")
     exec_layers = prof.get("attention", (0, 0))[1] / prof_steps
     per_layer_kernels = sum(prof.get(k, (0, 0))[1] for k in per_layer) / max(exec_layers * prof_steps, 1)
     graph_extra = max(s.n_layers - exec_layers, 0) * per_layer_kernels

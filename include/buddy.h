@@ -335,7 +335,6 @@ enum {
   BUDDY_PROF_ATTENTION, BUDDY_PROF_GEMM_O, BUDDY_PROF_GEMM_GATE_UP, BUDDY_PROF_GEMM_DOWN,
   BUDDY_PROF_ROUTE, BUDDY_PROF_COMPACT, BUDDY_PROF_OTHER,
   BUDDY_PROF_GEMM_FIXUP,   /* split-K sums + epilogues of the GEMMs (larger batches) */
-  BUDDY_PROF_ATTN_MERGE,   /* span merge of the tensor-core attention */
   BUDDY_PROF_PF_GEMM,      /* prefill: projections (tcgen05, M-tiled) */
   BUDDY_PROF_PF_ATTENTION, /* prefill: causal attention */
   BUDDY_PROF_PF_OTHER,     /* prefill: RMSNorm, zero fill, advance */

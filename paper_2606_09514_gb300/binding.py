@@ -26,7 +26,7 @@ EXPORTED = ["buddy_create", "buddy_destroy", "buddy_set_weights", "buddy_kv_appe
             "buddy_set_wait_limit"]
 PROF_CLASSES = ["check", "rmsnorm", "gemm_qkv", "qkv_finalize", "attention", "gemm_o", "gemm_gate_up",
                 "gemm_down", "route", "compact", "other", "gemm_fixup",
-                "attn_merge", "pf_gemm", "pf_attention", "pf_other"]
+                "pf_gemm", "pf_attention", "pf_other"]
 
 c_p = ctypes.c_void_p
 c_i32 = ctypes.c_int32
@@ -271,7 +271,7 @@ class Context:
         v = (c_i32 * 4)()
         _check(self.lib.buddy_get_paths(self.handle, v, 4), "buddy_get_paths")
         return {"gemm": "tcgen05 bf16 (TMA, TMEM)" if v[0] else "CUDA-core fp32",
-                "attention": ["CUDA-core", "mma.sync tensor-core, span merge kernel",
+                "attention": ["CUDA-core", "mma.sync tensor-core, warp shares over the GPU (in-kernel span merge)",
                               "mma.sync tensor-core, one cluster per stream (DSMEM merge)"][v[1]],
                 "rmsnorm": "inside the QKV and gate/up GEMMs" if v[2] else "separate kernel",
                 "split_k_fixup": "separate kernel" if v[3] else "last-arriving CTA"}

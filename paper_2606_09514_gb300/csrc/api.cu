@@ -55,7 +55,7 @@ static void free_ctx(buddy_ctx* x) {
   void* ptrs[] = {c.rope_cos, c.rope_sin, c.status, c.xn, c.act, c.attn_out, c.qkv, c.q,
                   c.attn_m, c.attn_l, c.attn_acc, c.attn_ctr, c.dm_u, c.dm_x, c.mask, c.sel, c.scores, c.rows,
                   c.count, c.h_in_stage, c.h_out_stage, c.k_stage, c.mask_stage, c.xn_lo, c.act_lo, c.attn_lo,
-                  c.gemm_ws, c.gemm_ctr, c.attn_meta, c.pf_xn, c.pf_xn_lo, c.pf_q, c.pf_attn, c.pf_attn_lo,
+                  c.gemm_ws, c.gemm_ctr, c.pf_xn, c.pf_xn_lo, c.pf_q, c.pf_attn, c.pf_attn_lo,
                   c.pf_act, c.pf_act_lo, c.pf_tok_seq, c.pf_tok_t, c.pf_tok_pos, c.pf_rows, c.pf_items,
                   c.pf_n_tok, c.pf_tok_end, c.pf_cnt, c.pf_hlast};
   for (void* p : ptrs)
@@ -133,7 +133,7 @@ extern "C" int buddy_create(const buddy_config* cfg, buddy_ctx** out) {
       (e = dalloc(&c.attn_m, B * c.nq * c.attn_max_chunks)) ||
       (e = dalloc(&c.attn_l, B * c.nq * c.attn_max_chunks)) ||
       (e = dalloc(&c.attn_acc, B * c.nq * c.attn_max_chunks * c.hd)) ||
-      (e = dalloc(&c.attn_ctr, B * c.nkv)) || (e = dalloc(&c.attn_meta, B + 2)) ||
+      (e = dalloc(&c.attn_ctr, B * c.nkv)) ||
       (e = dalloc(&c.dm_u, (size_t)kRouteZSlots * B * c.r)) || (e = dalloc(&c.dm_x, B * 2 * c.d)) ||
       (e = dalloc(&c.mask, B * c.L)) ||
       (e = dalloc(&c.sel, B * c.Lm)) || (e = dalloc(&c.scores, B * c.Lm)) ||
@@ -297,7 +297,7 @@ extern "C" const char* buddy_profile_class_name(int32_t cls) {
   static const char* names[BUDDY_PROF_NCLASS] = {"check", "rmsnorm", "gemm_qkv", "qkv_finalize",
                                                  "attention", "gemm_o", "gemm_gate_up", "gemm_down",
                                                  "route", "compact", "other", "gemm_fixup",
-                                                 "attn_merge", "pf_gemm", "pf_attention", "pf_other"};
+                                                 "pf_gemm", "pf_attention", "pf_other"};
   return (cls >= 0 && cls < BUDDY_PROF_NCLASS) ? names[cls] : "unknown";
 }
 
@@ -409,14 +409,8 @@ static GemmArgs down_args(const Ctx& c, int l, RowSel sel, float* H, bool split)
 
 static void enqueue_attention(Ctx& c, const buddy_kv_state& kv, int l, RowSel sel, bool split, cudaStream_t s,
                               bool prof) {
-  {
-    ProfScope p(c, s, BUDDY_PROF_ATTENTION, 1, prof);
-    launch_attention(c, sel, kv, l, c.q, c.attn_out, split ? c.attn_lo : nullptr, s);
-  }
-  if (attention_tc(c) && !attention_cl(c)) {
-    ProfScope p(c, s, BUDDY_PROF_ATTN_MERGE, 1, prof);
-    launch_attention_merge(c, sel, c.attn_out, split ? c.attn_lo : nullptr, s);
-  }
+  ProfScope p(c, s, BUDDY_PROF_ATTENTION, 1, prof);
+  launch_attention(c, sel, kv, l, c.q, c.attn_out, split ? c.attn_lo : nullptr, s);
 }
 
 // One decoder block, one launch per GEMM.

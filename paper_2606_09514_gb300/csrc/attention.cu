@@ -5,8 +5,9 @@
 //
 // Two work loops:
 //   * bf16 caches (G <= 8): the tensor-core loop of attn_tc.cuh (warp shares
-//     of the concatenated position streams, mma.sync contractions) and its
-//     span-merge kernel;
+//     of the concatenated position streams, mma.sync contractions, span
+//     partials merged by the warp that completes a stream), or at a few rows
+//     the cluster loop of attn_cl.cu;
 //   * fp32 caches: the CUDA-core
 //     loop of attn_common.cuh.  Its work items are (row, KV head, span of P
 //     positions); P is derived on the device from the total number of
@@ -37,13 +38,6 @@ __global__ void __launch_bounds__(kTcaThreads) attn_tc_kernel(AttnArgs<bf16> A) 
   attn_tc_run<HD, SPLIT>(A, blockIdx.x, gridDim.x, smraw, sc, true);
 }
 
-template <int HD>
-__global__ void __launch_bounds__(kTcaMergeThreads) attn_tc_merge_kernel(AttnArgs<bf16> A) {
-  pdl_wait();
-  pdl_trigger();
-  attn_tc_merge_run<HD>(A);
-}
-
 // bf16 caches with at most 8 query heads per KV head: the tensor-core loop
 template <int HD, bool SPLIT>
 static void attn_tc_impl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q, void* out,
@@ -61,16 +55,8 @@ static void attn_tc_impl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int
   const int grid = c.num_sms * std::max(1, std::min(occ, 4));
   AttnArgs<bf16> A{q, sel.rows, sel.count, sel.n, c.nq, c.nkv, cache_len(c, kv, layer), kv.seq_off, kv.cap,
                    (const bf16*)kv.k_cache[layer], (const bf16*)kv.v_cache[layer], c.attn_max_chunks, c.attn_m,
-                   c.attn_l, c.attn_acc, c.attn_ctr, (bf16*)out, (bf16*)out_lo, c.status, c.attn_meta};
+                   c.attn_l, c.attn_acc, c.attn_ctr, (bf16*)out, (bf16*)out_lo, c.status};
   launch_k(attn_tc_kernel<HD, SPLIT>, grid, kTcaThreads, smem, s, c.pdl, A);
-}
-
-template <int HD>
-static void attn_tc_merge_impl(const Ctx& c, RowSel sel, void* out, void* out_lo, cudaStream_t s) {
-  AttnArgs<bf16> A{nullptr, sel.rows, sel.count, sel.n, c.nq, c.nkv, nullptr, nullptr, nullptr, nullptr, nullptr,
-                   c.attn_max_chunks, c.attn_m, c.attn_l, c.attn_acc, nullptr, (bf16*)out, (bf16*)out_lo,
-                   c.status, c.attn_meta};
-  launch_k(attn_tc_merge_kernel<HD>, c.maxB * c.nkv, kTcaMergeThreads, 0, s, c.pdl, A);
 }
 
 template <typename T, int HD, int GP>
@@ -124,15 +110,10 @@ int attention_max_spans(int max_pos) {
 }
 
 // bf16 caches with at most 8 query heads per KV head whose per-row tables fit
-// next to the chunk buffers take the tensor-core loop (and its merge kernel)
+// next to the chunk buffers take the tensor-core loop
 bool attention_tc(const Ctx& c) {
   return c.dtype == BUDDY_DTYPE_BF16 && c.nq / c.nkv <= 8 &&
          attn_tc_smem_bytes(c.hd, c.maxB) <= (size_t)kTcaSmemLimit;
-}
-
-void launch_attention_merge(const Ctx& c, RowSel sel, void* out, void* out_lo, cudaStream_t s) {
-  if (c.hd == 128) attn_tc_merge_impl<128>(c, sel, out, out_lo, s);
-  else attn_tc_merge_impl<64>(c, sel, out, out_lo, s);
 }
 
 void launch_attention(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q,

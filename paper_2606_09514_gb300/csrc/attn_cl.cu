@@ -444,7 +444,7 @@ static void attn_cl_impl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int
   const int C = cl_size<HD, SPLIT>(sel.n * c.nkv);
   AttnArgs<bf16> A{q, sel.rows, sel.count, sel.n, c.nq, c.nkv, cache_len(c, kv, layer), kv.seq_off, kv.cap,
                    (const bf16*)kv.k_cache[layer], (const bf16*)kv.v_cache[layer], 0, nullptr, nullptr, nullptr,
-                   nullptr, (bf16*)out, (bf16*)out_lo, c.status, nullptr};
+                   nullptr, (bf16*)out, (bf16*)out_lo, c.status};
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(C, sel.n * c.nkv, 1);
   cfg.blockDim = dim3(kClThreads, 1, 1);

@@ -82,7 +82,6 @@ struct AttnArgs {
   T* out;
   T* out_lo;
   const int32_t* status;
-  int32_t* meta;   // tensor-core loop: row prefix and share for its merge kernel
 };
 
 // Dynamic shared memory used by attn_run (bytes): double-buffered K (rows

@@ -8,13 +8,12 @@
 // cover several short ones; the piece of a stream that one warp holds is a
 // span.  A stream held by one warp is written out directly; otherwise every
 // warp writes its span's partial (running max, sum of exponentials,
-// unnormalised output), and the partials are merged in span order
-// (deterministic): for at most kTcaWarpMerge spans by the warp that completes
-// the stream last (an arrival counter per stream), for more (small batches,
-// long rows) by attn_tc_merge_kernel, launched right after, one CTA per
-// stream.  Because warps never wait for each other, each streams its share
-// without a break: the copies of the next span are in flight while the
-// current one finishes (or merges).
+// unnormalised output), and the warp that completes the stream last (an
+// arrival counter per stream) merges the partials in span order
+// (deterministic), kTcaWarpMerge spans' loads at a time.  Because warps never
+// wait for each other, each streams its share without a break: the copies of
+// the next span are in flight while the current one finishes (or merges), and
+// no second kernel is needed.
 //
 // Inside a share a warp walks chunks of up to kTcaChunk positions (never
 // crossing a stream end):
@@ -50,8 +49,7 @@ constexpr int kTcaWarps = 4;
 constexpr int kTcaThreads = 32 * kTcaWarps;
 constexpr int kTcaStages = 3;     // chunk buffers per warp (kTcaStages - 1 in flight)
 constexpr int kTcaMinShare = 2 * kTcaChunk;   // positions of a warp's share, at least
-constexpr int kTcaMergeThreads = 256;         // merge kernel: one CTA per stream
-constexpr int kTcaWarpMerge = 4;              // streams of at most this many spans merge in the kernel
+constexpr int kTcaWarpMerge = 4;              // span partials loaded at a time by the merging warp
 
 template <int HD>
 __host__ __device__ constexpr size_t attn_tc_smem_fixed() {
@@ -113,10 +111,12 @@ __device__ __forceinline__ float exp2a(float x) {
 
 }  // namespace tca
 
-// Merge of a (row j, KV head g)'s nsp <= kTcaWarpMerge span partials by one
-// warp: lane -> (head, four channels) per round of 32 lanes; two rounds'
-// partials (every span's output, max and sum) are loaded at once, then each
-// output is sum_s 2^(m_s - M) o_s / sum_s 2^(m_s - M) l_s, in span order.
+// Merge of a (row j, KV head g)'s nsp span partials by one warp: lane ->
+// (head, four channels) per round of 32 lanes.  For two rounds at a time the
+// partials (output, max and sum) of kTcaWarpMerge spans are loaded at once and
+// folded into a running max M, sum L and output O in span order (a group
+// raising M rescales what came before by 2^(M_old - M_new)); the result is
+// O / L, i.e. sum_s 2^(m_s - M) o_s / sum_s 2^(m_s - M) l_s.
 template <int HD>
 __device__ __forceinline__ void attn_tc_warp_merge(const AttnArgs<bf16>& A, int j, int g, int nsp, size_t obase,
                                                    int lane) {
@@ -127,18 +127,50 @@ __device__ __forceinline__ void attn_tc_warp_merge(const AttnArgs<bf16>& A, int 
   const size_t hb0 = ((size_t)j * A.nq + (size_t)g * G) * ms;
   const int hsub = lane / Q, e0 = (lane % Q) * 4;
   for (int r0 = 0; r0 * HPR < G; r0 += 2) {
-    float4 v[2][NS];
-    float mv[2][NS], lv[2][NS];
+    float M[2] = {-INFINITY, -INFINITY}, L[2] = {0.f, 0.f};
+    float4 acc[2] = {make_float4(0.f, 0.f, 0.f, 0.f), make_float4(0.f, 0.f, 0.f, 0.f)};
+    for (int s0 = 0; s0 < nsp; s0 += NS) {
+      float4 v[2][NS];
+      float mv[2][NS], lv[2][NS];
 #pragma unroll
-    for (int u = 0; u < 2; ++u) {
-      const int h = (r0 + u) * HPR + hsub;
+      for (int u = 0; u < 2; ++u) {
+        const int h = (r0 + u) * HPR + hsub;
 #pragma unroll
-      for (int s = 0; s < NS; ++s) {
-        if (h < G && s < nsp) {
-          const size_t slot = hb0 + (size_t)h * ms + s;
-          v[u][s] = __ldcg(reinterpret_cast<const float4*>(A.part_acc + slot * HD + e0));
-          mv[u][s] = __ldcg(A.part_m + slot);
-          lv[u][s] = __ldcg(A.part_l + slot);
+        for (int s = 0; s < NS; ++s) {
+          if (h < G && s0 + s < nsp) {
+            const size_t slot = hb0 + (size_t)h * ms + s0 + s;
+            v[u][s] = __ldcg(reinterpret_cast<const float4*>(A.part_acc + slot * HD + e0));
+            mv[u][s] = __ldcg(A.part_m + slot);
+            lv[u][s] = __ldcg(A.part_l + slot);
+          }
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int h = (r0 + u) * HPR + hsub;
+        if (h >= G) continue;
+        float mn = M[u];
+#pragma unroll
+        for (int s = 0; s < NS; ++s)
+          if (s0 + s < nsp) mn = fmaxf(mn, mv[u][s]);
+        // span maxima are finite, so mn is; 2^(-inf) = 0 on the first group
+        const float sc = tca::exp2a(M[u] - mn);
+        M[u] = mn;
+        L[u] *= sc;
+        acc[u].x *= sc;
+        acc[u].y *= sc;
+        acc[u].z *= sc;
+        acc[u].w *= sc;
+#pragma unroll
+        for (int s = 0; s < NS; ++s) {
+          if (s0 + s < nsp) {
+            const float w = tca::exp2a(mv[u][s] - mn);
+            L[u] += w * lv[u][s];
+            acc[u].x += w * v[u][s].x;
+            acc[u].y += w * v[u][s].y;
+            acc[u].z += w * v[u][s].z;
+            acc[u].w += w * v[u][s].w;
+          }
         }
       }
     }
@@ -146,29 +178,12 @@ __device__ __forceinline__ void attn_tc_warp_merge(const AttnArgs<bf16>& A, int 
     for (int u = 0; u < 2; ++u) {
       const int h = (r0 + u) * HPR + hsub;
       if (h >= G) continue;
-      float M = mv[u][0];
-#pragma unroll
-      for (int s = 1; s < NS; ++s)
-        if (s < nsp) M = fmaxf(M, mv[u][s]);
-      float L = 0.f;
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-      for (int s = 0; s < NS; ++s) {
-        if (s < nsp) {
-          const float w = tca::exp2a(mv[u][s] - M);
-          L += w * lv[u][s];
-          acc.x += w * v[u][s].x;
-          acc.y += w * v[u][s].y;
-          acc.z += w * v[u][s].z;
-          acc.w += w * v[u][s].w;
-        }
-      }
-      const float inv = 1.f / L;
+      const float inv = 1.f / L[u];
       const size_t o = obase + (size_t)h * HD + e0;
-      store_out(A.out, A.out_lo, o + 0, acc.x * inv);
-      store_out(A.out, A.out_lo, o + 1, acc.y * inv);
-      store_out(A.out, A.out_lo, o + 2, acc.z * inv);
-      store_out(A.out, A.out_lo, o + 3, acc.w * inv);
+      store_out(A.out, A.out_lo, o + 0, acc[u].x * inv);
+      store_out(A.out, A.out_lo, o + 1, acc[u].y * inv);
+      store_out(A.out, A.out_lo, o + 2, acc[u].z * inv);
+      store_out(A.out, A.out_lo, o + 3, acc[u].w * inv);
     }
   }
 }
@@ -235,15 +250,6 @@ __device__ __forceinline__ void attn_tc_run(const AttnArgs<bf16>& A, int cta, in
       const int nw = ncta * kTcaWarps;
       const int even = (carry + nw - 1) / nw;
       sc[0] = max(kTcaMinShare, (even + CH - 1) / CH * CH);
-    }
-    // the merge kernel's copy of the prefix and the share
-    if (cta == 0) {
-      __syncwarp();
-      for (int j = lane; j < m; j += 32) A.meta[j + 1] = pref[j + 1];
-      if (lane == 0) {
-        A.meta[0] = 0;
-        A.meta[m + 1] = sc[0];
-      }
     }
   }
   __syncthreads();
@@ -500,7 +506,7 @@ __device__ __forceinline__ void attn_tc_run(const AttnArgs<bf16>& A, int cta, in
             }
           }
         }
-      } else {   // a partial for attn_tc_merge_kernel
+      } else {   // a partial, merged by the warp that completes the stream
         const int sp = gw - first;
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
@@ -518,40 +524,22 @@ __device__ __forceinline__ void attn_tc_run(const AttnArgs<bf16>& A, int cta, in
             }
           }
         }
-        if (nsp <= kTcaWarpMerge) {
-          // the partial is visible before the arrival is counted; the warp
-          // that completes the stream merges (and re-arms the counter)
-          __syncwarp();
-          int last = 0;
-          if (lane == 0) {
-            int32_t* ctr = A.ctr + cs.j * nkv + cs.g;
-            const int old = ptx::atom_add_acq_rel(ctr, 1);
-            last = old == nsp - 1;
-            if (last) *ctr = 0;   // re-armed for a later launch
-          }
-          last = __shfl_sync(0xffffffffu, last, 0);
-          __syncwarp();
-          if (last) attn_tc_warp_merge<HD>(A, cs.j, cs.g, nsp, obase, lane);
+        // the partial is visible before the arrival is counted; the warp
+        // that completes the stream merges (and re-arms the counter)
+        __syncwarp();
+        int last = 0;
+        if (lane == 0) {
+          int32_t* ctr = A.ctr + cs.j * nkv + cs.g;
+          const int old = ptx::atom_add_acq_rel(ctr, 1);
+          last = old == nsp - 1;
+          if (last) *ctr = 0;   // re-armed for a later launch
         }
+        last = __shfl_sync(0xffffffffu, last, 0);
+        __syncwarp();
+        if (last) attn_tc_warp_merge<HD>(A, cs.j, cs.g, nsp, obase, lane);
       }
     }
   }
-}
-
-// Merge of the span partials of stream (row j, KV head g) = (blockIdx.x /
-// nkv, blockIdx.x % nkv), in span order, for streams the attention kernel cut
-// into more than kTcaWarpMerge spans.
-template <int HD>
-__device__ __forceinline__ void attn_tc_merge_run(const AttnArgs<bf16>& A) {
-  const int m = A.count ? *A.count : A.n;
-  const int j = blockIdx.x / A.nkv, g = blockIdx.x - j * A.nkv;
-  if (j >= m || *reinterpret_cast<const volatile int32_t*>(A.status + 1) != 0) return;
-  const int np = (A.meta[j + 1] - A.meta[j]) / A.nkv, share = A.meta[m + 1];
-  const int S0 = A.meta[j] + g * np;
-  const int nsp = (S0 + np - 1) / share - S0 / share + 1;
-  if (nsp <= kTcaWarpMerge) return;   // written out, or merged in the attention kernel
-  const size_t obase = ((size_t)j * A.nq + (size_t)g * (A.nq / A.nkv)) * HD;
-  attn_span_merge<bf16, HD, kTcaMergeThreads, true>(A, j, g, nsp, obase, threadIdx.x);
 }
 
 }  // namespace buddy

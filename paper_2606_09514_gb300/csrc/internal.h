@@ -122,11 +122,10 @@ void launch_qkv_finalize(const Ctx& c, const float* qkv, const float* bias, RowS
 void launch_attention(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q,
                       void* attn_out, void* attn_lo, cudaStream_t s);   // attention.cu
 int attention_max_spans(int max_pos);   // span partials per (row, query head)
-bool attention_tc(const Ctx& c);         // tensor-core loop: launch_attention_merge follows
-bool attention_cl(const Ctx& c);         // small batches: one cluster per stream, no merge kernel (attn_cl.cu)
+bool attention_tc(const Ctx& c);         // tensor-core loop over the whole GPU
+bool attention_cl(const Ctx& c);         // small batches: one cluster per stream (attn_cl.cu)
 void launch_attention_cl(const Ctx& c, RowSel sel, const buddy_kv_state& kv, int layer, const float* q, void* out,
                          void* out_lo, cudaStream_t s);
-void launch_attention_merge(const Ctx& c, RowSel sel, void* out, void* out_lo, cudaStream_t s);
 void launch_route(const Ctx& c, int B, const float* h1, const float* pool, const int32_t* len,
                   int len_bias, const int32_t* k, uint8_t* mask, int32_t* sel, float* scores,
                   cudaStream_t s);
@@ -195,7 +194,6 @@ struct Ctx {
   float* attn_l = nullptr;
   float* attn_acc = nullptr;   // [maxB, nq, max_chunks, hd]
   int32_t* attn_ctr = nullptr; // [maxB, nkv] chunk arrivals (self-resetting)
-  int32_t* attn_meta = nullptr;   // [maxB + 2] row prefix and share (tensor-core attention)
   float* dm_u = nullptr;       // [kRouteZSlots, maxB, r + predictor hidden] partial sums
   float* dm_x = nullptr;       // [maxB, 2d] router inputs (larger batches)
   uint8_t* mask = nullptr;     // [maxB, L]
