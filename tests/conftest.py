@@ -10,4 +10,3 @@ if ROOT not in sys.path:
 
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (sm_103a) and the built libbuddy")
-    config.addinivalue_line("markers", "slow: full-size workload")
